@@ -1,0 +1,108 @@
+"""Pins for oracle.numerics and oracle.philox against closed forms, library routines and
+published known-answer vectors."""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle.numerics import bf16, rmsnorm, rope, silu
+from oracle.philox import (draw_u32, gumbel, philox4x32_10, u_accept, u_open)
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def test_bf16_matches_torch_rne():
+    rng = np.random.default_rng(0)
+    x = np.concatenate([rng.standard_normal(20000) * 10.0 ** rng.integers(-6, 6, 20000),
+                        [0.0, 1.0, -1.0, 1 + 2 ** -8, 1 + 3 * 2 ** -8, -(1 + 2 ** -8)]]).astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(bf16(x.astype(np.float64)), ref)
+
+
+def test_bf16_ties_to_even():
+    assert bf16(1 + 2 ** -8) == 1.0               # halfway, even neighbour is 1.0
+    assert bf16(1 + 3 * 2 ** -8) == 1 + 2 ** -6    # halfway, even neighbour is above
+    assert bf16(1 + 2 ** -8 + 2 ** -20) == 1 + 2 ** -7
+
+
+def test_rmsnorm_closed_form():
+    h = np.full((3, 64), -2.5)
+    g = np.linspace(0.5, 1.5, 64)
+    out = rmsnorm(h, g, 1e-6)
+    np.testing.assert_allclose(out, np.broadcast_to(-2.5 / np.sqrt(6.25 + 1e-6) * g[None, :], out.shape), rtol=1e-15)
+    # torch's rms_norm as an independent routine
+    x = np.random.default_rng(1).standard_normal((5, 32))
+    ref = torch.nn.functional.rms_norm(torch.from_numpy(x), (32,), torch.from_numpy(g[:32]), eps=1e-6).numpy()
+    np.testing.assert_allclose(rmsnorm(x, g[:32], 1e-6), ref, rtol=1e-12)
+
+
+def test_rope_identity_norm_and_relative_position():
+    rng = np.random.default_rng(2)
+    q = rng.standard_normal((1, 2, 16))
+    k = rng.standard_normal((1, 2, 16))
+    np.testing.assert_allclose(rope(q, np.array([0]), 1e4), q, rtol=0, atol=0)
+    r = rope(q, np.array([37]), 1e4)
+    # rotation of pairs (i, i + hd/2) preserves each pair's norm
+    n0 = q[..., :8] ** 2 + q[..., 8:] ** 2
+    n1 = r[..., :8] ** 2 + r[..., 8:] ** 2
+    np.testing.assert_allclose(n0, n1, rtol=1e-12)
+    # <rope(q, m), rope(k, n)> depends only on m - n
+    a = np.sum(rope(q, np.array([10]), 1e4) * rope(k, np.array([3]), 1e4))
+    b = np.sum(rope(q, np.array([107]), 1e4) * rope(k, np.array([100]), 1e4))
+    np.testing.assert_allclose(a, b, rtol=1e-10)
+    # pair (0, hd/2) rotates by exactly pos radians (frequency theta^0 = 1)
+    e = np.zeros((1, 1, 16)); e[0, 0, 0] = 1.0
+    r = rope(e, np.array([0.75]), 1e4)
+    np.testing.assert_allclose([r[0, 0, 0], r[0, 0, 8]], [np.cos(0.75), np.sin(0.75)], rtol=1e-14)
+
+
+def test_silu_library():
+    x = np.linspace(-20, 20, 101)
+    np.testing.assert_allclose(silu(x), torch.nn.functional.silu(torch.from_numpy(x)).numpy(), rtol=1e-12)
+
+
+def _read_kat():
+    rows = []
+    with open(os.path.join(GOLD, "philox4x32_10_kat.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                rows.append([int(t, 16) for t in line.split()])
+    return rows
+
+
+def test_philox_known_answers():
+    for r in _read_kat():
+        out = philox4x32_10(*r[:6])
+        assert [int(x) for x in out] == r[6:]
+
+
+def test_philox_uniform_statistics():
+    w = draw_u32(1234, 1, 2, 3, 4, np.arange(200000))
+    u = u_accept(w)
+    assert u.min() > 0 and u.max() <= 1.0
+    assert abs(u.mean() - 0.5) < 4 * np.sqrt(1 / 12 / u.size)
+    hist = np.bincount((w >> np.uint32(24)).astype(np.int64), minlength=256)
+    e = u.size / 256
+    chi2 = np.sum((hist - e) ** 2 / e)
+    assert chi2 < 255 + 6 * np.sqrt(2 * 255)
+    # every value is an exact multiple of 2**-24
+    assert np.all(np.floor(u * 2 ** 24) == u * 2 ** 24)
+    uo = u_open(w)
+    assert uo.min() > 0 and uo.max() < 1
+
+
+def test_philox_streams_differ():
+    a = draw_u32(0, 0, 1, 0, 0, np.arange(64))
+    b = draw_u32(0, 1, 1, 0, 0, np.arange(64))
+    c = draw_u32(0, 0, 1, 0, 1, np.arange(64))
+    assert not np.array_equal(a, b) and not np.array_equal(a, c)
+    # word selection: draws 4i..4i+3 are the four outputs of one counter
+    words = philox4x32_10(0, 1, 0, 0, 0, 0)
+    np.testing.assert_array_equal(a[:4], np.array([int(x) for x in words], dtype=np.uint32))
+
+
+def test_gumbel_moments():
+    g = gumbel(draw_u32(7, 3, 1, 0, 0, np.arange(400000))).astype(np.float64)
+    assert abs(g.mean() - 0.5772156649) < 4 * np.sqrt(np.pi ** 2 / 6 / g.size)
+    assert abs(g.var() - np.pi ** 2 / 6) < 0.02
