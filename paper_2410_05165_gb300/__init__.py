@@ -1,0 +1,12 @@
+"""GB300 (sm_103a) implementation of the AtSpeed verification call (arXiv 2410.05165).
+
+The CUDA library ``_build/libatspeed.so`` (sources in ``csrc/``, C ABI in ``include/atspeed.h``)
+does all the work; ``binding`` marshals torch tensors into its calls.
+"""
+from .binding import (AtSpeedError, Context, DecodeOpts, EXPORTS, LIB_PATH, NORM_MASKED, PLAIN_SAMPLE, PLAIN_TOPK,
+                      RELAXED, SD_RELAXED, SD_STRICT, STRICT, load, op_attention, op_gemm, op_gemm_swiglu, op_rmsnorm,
+                      opts, weights_to_device)
+
+__all__ = ["AtSpeedError", "Context", "DecodeOpts", "EXPORTS", "LIB_PATH", "NORM_MASKED", "PLAIN_SAMPLE",
+           "PLAIN_TOPK", "RELAXED", "SD_RELAXED", "SD_STRICT", "STRICT", "load", "op_attention", "op_gemm",
+           "op_gemm_swiglu", "op_rmsnorm", "opts", "weights_to_device"]

@@ -1,0 +1,498 @@
+// Weight-streaming GEMM for sm_103a: TMA -> shared memory (128B swizzle) -> tcgen05.mma with the
+// fp32 accumulator in TMEM -> tcgen05.ld epilogue with fused QKV+RoPE+KV-store / SwiGLU /
+// residual-add / plain stores.
+//
+// Decomposition ("stream-K"): the work units are (tile, 64-wide k-block) pairs, tile = (weight-row
+// tile of 128, token tile of BN), ordered weight-tile-major.  A persistent grid of one CTA per SM
+// takes equal contiguous ranges of units, so every SM streams the same number of weight bytes
+// whatever the matrix shape.  A tile whose k-range spans several CTAs is reduced through an fp32
+// workspace by the last CTA to finish it (fixed summation order, hence deterministic), which then
+// runs the fused epilogue.  The partition depends only on (M, K, tokens rounded to the tile and
+// the grid), so a token's output does not depend on which other tokens share the call.
+//
+// Roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM allocator + MMA issuer, warps 2-5 =
+// epilogue (TMEM lane quadrant = warp % 4).  Two TMEM accumulators alternate between segments so
+// the next segment's MMAs overlap the previous segment's epilogue.
+#include <cudaTypedefs.h>
+#include <stdio.h>
+
+#include "common.cuh"
+#include "gemm.cuh"
+
+namespace atspeed {
+
+namespace {
+
+constexpr int BK = 64;            // bf16 elements per 128-byte swizzle row
+constexpr int BM = 128;           // weight rows per tile (MMA M)
+constexpr int WS_SLOT_FLOATS = 256 * 128;
+constexpr int MAX_TILES = 1 << 16;
+
+template <int BN>
+struct Cfg {
+  static constexpr int STAGES = (BN == 128) ? 6 : 4;
+  static constexpr int A_BYTES = BM * 128;
+  static constexpr int B_BYTES = BN * 128;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGING_FLOATS = 32 * BM;
+  static constexpr int BAR_BYTES = 256;
+  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_FLOATS * 4 + BAR_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;
+};
+
+struct KParams {
+  GemmArgs a;
+  int m_tiles, n_tiles, kb;
+  long long U;
+  int G;
+  int up_row0;
+  float* ws;
+  int* counters;
+  unsigned int* err;
+};
+
+__device__ __forceinline__ long long unit_start(long long c, long long U, int G) { return c * U / G; }
+__device__ __forceinline__ int unit_owner(long long u, long long U, int G) {
+  return (int)(((u + 1) * (long long)G - 1) / U);
+}
+
+template <int BN, int EPI>
+__device__ __forceinline__ void epi_chunk(const KParams& p, const float* st, int m_tile, int n_tile, int ch,
+                                          int ep_tid) {
+  const GemmArgs& a = p.a;
+  const int tok0 = n_tile * BN + ch * 32;
+  if constexpr (EPI == EPI_SWIGLU) {
+    for (int idx = ep_tid; idx < 32 * 64; idx += 128) {
+      const int n = idx >> 6, i = idx & 63;
+      const int tok = tok0 + n;
+      if (tok >= a.T) continue;
+      const float g = st[n * BM + i];
+      const float u = st[n * BM + 64 + i];
+      const float s = g / (1.0f + expf(-g));
+      a.out_bf16[(size_t)tok * a.ldo + m_tile * 64 + i] = __float2bfloat16_rn(s * u);
+    }
+  } else {
+    for (int idx = ep_tid; idx < 32 * BM; idx += 128) {
+      const int n = idx >> 7, m = idx & 127;
+      const int tok = tok0 + n;
+      const int row = m_tile * BM + m;
+      if (tok >= a.T || row >= a.M) continue;
+      const float v = st[idx];
+      if constexpr (EPI == EPI_F32) {
+        a.out_f32[(size_t)tok * a.ldo + row] = v;
+      } else if constexpr (EPI == EPI_BF16) {
+        a.out_bf16[(size_t)tok * a.ldo + row] = __float2bfloat16_rn(v);
+      } else if constexpr (EPI == EPI_RESID) {
+        float* o = a.out_f32 + (size_t)tok * a.ldo + row;
+        *o = *o + v;
+      } else {  // EPI_QKV
+        const int d = a.d_model, hd = a.head_dim, half = hd >> 1;
+        const int region = row / d;
+        const int f = row - region * d;
+        if (region == 2) {
+          a.v_cache[(size_t)a.kv_row[tok] * d + f] = __float2bfloat16_rn(v);
+        } else {
+          const int i = f % hd;
+          const int ii = (i < half) ? i : i - half;
+          const size_t cs = (size_t)a.pos[tok] * half + ii;
+          const float cth = a.rope_cos[cs], sth = a.rope_sin[cs];
+          float out;
+          if (i < half) {
+            const float x2 = st[n * BM + m + half];
+            out = v * cth - x2 * sth;
+          } else {
+            const float x1 = st[n * BM + m - half];
+            out = v * cth + x1 * sth;
+          }
+          const __nv_bfloat16 ob = __float2bfloat16_rn(out);
+          if (region == 0)
+            a.q_out[(size_t)tok * d + f] = ob;
+          else
+            a.k_cache[(size_t)a.kv_row[tok] * d + f] = ob;
+        }
+      }
+    }
+  }
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(192, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const KParams p) {
+  using C = Cfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  float* staging = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(staging + C::STAGING_FLOATS);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* tfull = empty + C::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* mma_done = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  int* flag = reinterpret_cast<int*>(tmem_slot + 1);
+  int* failed = flag + 1;
+  int* last_fill = failed + 1;  // [STAGES]: parity of the last fill issued per stage, -1 if none
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = blockIdx.x;
+  const long long u0 = unit_start(c, p.U, p.G), u1 = unit_start(c + 1, p.U, p.G);
+  const int kb = p.kb;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+      last_fill[s] = -1;
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 4);
+    }
+    mbar_init(mma_done, 1);
+    *failed = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  pdl_launch_dependents();
+
+  if (warp == 0) {
+    if (lane == 0 && u1 > u0) {
+      // ------------------------------------------------------------------ TMA producer
+      tma_prefetch_desc(&tmA);
+      tma_prefetch_desc(&tmB);
+      const uint64_t pol_w = policy_evict_first();   // weights: streamed once
+      const uint64_t pol_x = policy_evict_last();    // activations: re-read by every CTA
+      const long long total = u1 - u0;
+      const int npre = (int)(total < C::STAGES ? total : C::STAGES);
+      auto a_rows = [&](long long u, int& r0, int& r1, int& xk, int& brow) {
+        const int tile = (int)(u / kb), kbi = (int)(u % kb);
+        const int mt = tile / p.n_tiles, nt = tile % p.n_tiles;
+        if (EPI == EPI_SWIGLU) {
+          r0 = mt * 64;
+          r1 = p.up_row0 + mt * 64;
+        } else {
+          r0 = mt * BM;
+          r1 = mt * BM + 64;
+        }
+        xk = kbi * BK;
+        brow = nt * BN;
+      };
+      // prologue: weights do not depend on the previous kernel, so fetch them before waiting
+      for (int i = 0; i < npre; ++i) {
+        int r0, r1, xk, brow;
+        a_rows(u0 + i, r0, r1, xk, brow);
+        uint8_t* sa = smem + i * C::STAGE_BYTES;
+        mbar_arrive_expect_tx(&full[i], C::STAGE_BYTES);
+        last_fill[i] = 0;
+        tma_load_2d(sa, &tmA, &full[i], xk, r0, pol_w);
+        tma_load_2d(sa + 8192, &tmA, &full[i], xk, r1, pol_w);
+      }
+      pdl_wait();
+      for (int i = 0; i < npre; ++i) {
+        int r0, r1, xk, brow;
+        a_rows(u0 + i, r0, r1, xk, brow);
+        tma_load_2d(smem + i * C::STAGE_BYTES + C::A_BYTES, &tmB, &full[i], xk, brow, pol_x);
+      }
+      int stage = npre % C::STAGES;
+      uint32_t phase = (npre == C::STAGES) ? 1u : 0u;
+      for (long long i = npre; i < total; ++i) {
+        if (!mbar_wait(&empty[stage], phase ^ 1u, p.err)) {
+          *failed = 1;
+          break;
+        }
+        int r0, r1, xk, brow;
+        a_rows(u0 + i, r0, r1, xk, brow);
+        uint8_t* sa = smem + stage * C::STAGE_BYTES;
+        mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
+        last_fill[stage] = (int)phase;
+        tma_load_2d(sa, &tmA, &full[stage], xk, r0, pol_w);
+        tma_load_2d(sa + 8192, &tmA, &full[stage], xk, r1, pol_w);
+        tma_load_2d(sa + C::A_BYTES, &tmB, &full[stage], xk, brow, pol_x);
+        if (++stage == C::STAGES) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && u1 > u0) {
+      // ------------------------------------------------------------------ MMA issuer
+      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int si = 0;
+      bool ok = true;
+      for (long long u = u0; u < u1 && ok; ++si) {
+        const int k0 = (int)(u % kb);
+        const long long len = (kb - k0) < (u1 - u) ? (kb - k0) : (u1 - u);
+        u += len;
+        const int acc = si & 1, use = si >> 1;
+        if (!mbar_wait(&tempty[acc], (uint32_t)(use & 1) ^ 1u, p.err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t dt = tmem_base + (uint32_t)(acc * BN);
+        for (long long j = 0; j < len; ++j) {
+          if (!mbar_wait(&full[stage], phase, p.err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * C::STAGE_BYTES);
+          const uint64_t ad = smem_desc_sw128(sa);
+          const uint64_t bd = smem_desc_sw128(sa + C::A_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            // advance the start address by kk * 32 bytes inside the 128-byte swizzle row
+            tc_mma_bf16(dt, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), idesc, (j > 0 || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(&empty[stage]);
+          if (++stage == C::STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        tc_commit(&tfull[acc]);
+      }
+      if (!ok) *failed = 1;
+      // drain: no MMA may still be running when TMEM is released
+      tc_commit(mma_done);
+      mbar_wait(mma_done, 0, p.err);
+    }
+  } else {
+    // -------------------------------------------------------------------- epilogue
+    const int q = warp & 3;
+    const int ep_tid = threadIdx.x - 64;
+    const int m = q * 32 + lane;
+    pdl_wait();
+    int si = 0;
+    for (long long u = u0; u < u1; ++si) {
+      const int tile = (int)(u / kb);
+      const int k0 = (int)(u % kb);
+      const long long len = (kb - k0) < (u1 - u) ? (kb - k0) : (u1 - u);
+      const int k1 = k0 + (int)len;
+      u += len;
+      const int acc = si & 1, use = si >> 1;
+      const bool got = mbar_wait(&tfull[acc], (uint32_t)(use & 1), p.err);
+      __syncwarp();
+      if (!got) {
+        *failed = 1;
+        break;
+      }
+      tc_fence_after();
+      const int m_tile = tile / p.n_tiles, n_tile = tile % p.n_tiles;
+      const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+      if (k0 == 0 && k1 == kb) {
+        for (int ch = 0; ch < BN / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tb + ch * 32, r);
+          tmem_ld_wait();
+          if (ch == BN / 32 - 1) {
+            tc_fence_before();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+          }
+#pragma unroll
+          for (int j = 0; j < 32; ++j) staging[j * BM + m] = __uint_as_float(r[j]);
+          named_bar_sync(1, 128);
+          epi_chunk<BN, EPI>(p, staging, m_tile, n_tile, ch, ep_tid);
+          named_bar_sync(1, 128);
+        }
+      } else {
+        const long long slot = (long long)c * 2 + (si == 0 ? 0 : 1);
+        float* wsl = p.ws + slot * WS_SLOT_FLOATS;
+        for (int ch = 0; ch < BN / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tb + ch * 32, r);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 32; ++j) __stcg(&wsl[(ch * 32 + j) * BM + m], __uint_as_float(r[j]));
+        }
+        tc_fence_before();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+        __threadfence();
+        named_bar_sync(1, 128);
+        const long long tu0 = (long long)tile * kb;
+        const int c_first = unit_owner(tu0, p.U, p.G);
+        const int c_last = unit_owner(tu0 + kb - 1, p.U, p.G);
+        const int parts = c_last - c_first + 1;
+        if (ep_tid == 0) {
+          const int old = atomicAdd(&p.counters[tile], 1);
+          const int last = (old == parts - 1);
+          if (last) {
+            p.counters[tile] = 0;
+            __threadfence();
+          }
+          *flag = last;
+        }
+        named_bar_sync(1, 128);
+        if (*flag) {
+          for (int ch = 0; ch < BN / 32; ++ch) {
+#pragma unroll 4
+            for (int j = 0; j < 32; ++j) {
+              float s = 0.0f;
+              for (int pi = 0; pi < parts; ++pi) {
+                const int cc = c_first + pi;
+                const long long sl = (long long)cc * 2 + (unit_start(cc, p.U, p.G) >= tu0 ? 0 : 1);
+                s += __ldcg(&p.ws[sl * WS_SLOT_FLOATS + (ch * 32 + j) * BM + m]);
+              }
+              staging[j * BM + m] = s;
+            }
+            named_bar_sync(1, 128);
+            epi_chunk<BN, EPI>(p, staging, m_tile, n_tile, ch, ep_tid);
+            named_bar_sync(1, 128);
+          }
+        }
+      }
+    }
+  }
+
+  __syncthreads();
+  if (*failed && threadIdx.x == 0) {
+    // make sure no TMA write is still headed for this CTA's shared memory
+    for (int s = 0; s < C::STAGES; ++s)
+      if (last_fill[s] >= 0) mbar_wait(&full[s], (uint32_t)last_fill[s], p.err);
+  }
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+bool make_map(CUtensorMap* m, const void* base, int inner, int rows, int box_rows, char* eb, size_t el) {
+  auto fn = encode_fn();
+  if (!fn) {
+    snprintf(eb, el, "cuTensorMapEncodeTiled unavailable");
+    return false;
+  }
+  cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)inner * 2};
+  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    snprintf(eb, el, "cuTensorMapEncodeTiled failed (%d): inner=%d rows=%d box_rows=%d", (int)r, inner, rows,
+             box_rows);
+    return false;
+  }
+  return true;
+}
+
+template <int BN, int EPI>
+cudaError_t launch_t(const CUtensorMap& ma, const CUtensorMap& mb, const KParams& kp, cudaStream_t st, bool pdl) {
+  using C = Cfg<BN>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kp.G);
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, gemm_kernel<BN, EPI>, ma, mb, kp);
+}
+
+template <int BN>
+cudaError_t launch_bn(EpiKind e, const CUtensorMap& ma, const CUtensorMap& mb, const KParams& kp, cudaStream_t st,
+                      bool pdl) {
+  switch (e) {
+    case EPI_F32: return launch_t<BN, EPI_F32>(ma, mb, kp, st, pdl);
+    case EPI_BF16: return launch_t<BN, EPI_BF16>(ma, mb, kp, st, pdl);
+    case EPI_RESID: return launch_t<BN, EPI_RESID>(ma, mb, kp, st, pdl);
+    case EPI_SWIGLU: return launch_t<BN, EPI_SWIGLU>(ma, mb, kp, st, pdl);
+    case EPI_QKV: return launch_t<BN, EPI_QKV>(ma, mb, kp, st, pdl);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+size_t gemm_ws_bytes(int grid) { return (size_t)2 * grid * WS_SLOT_FLOATS * sizeof(float); }
+int gemm_max_tiles() { return MAX_TILES; }
+
+int gemm_grid_size(int device) {
+  int sms = 0;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+  return sms > 0 ? sms : 1;
+}
+
+cudaError_t gemm_launch(const GemmArgs& a, const GemmScratch& s, int grid, cudaStream_t stream, bool pdl,
+                        char* eb, size_t el) {
+  if (a.K <= 0 || a.K % BK != 0 || a.M <= 0 || a.T <= 0) {
+    snprintf(eb, el, "gemm: bad shape M=%d K=%d T=%d", a.M, a.K, a.T);
+    return cudaErrorInvalidValue;
+  }
+  const int BN = a.T <= 128 ? 128 : 256;
+  KParams kp;
+  kp.a = a;
+  kp.n_tiles = (a.T + BN - 1) / BN;
+  if (a.X_rows < kp.n_tiles * BN) {
+    snprintf(eb, el, "gemm: X has %d rows, needs %d", a.X_rows, kp.n_tiles * BN);
+    return cudaErrorInvalidValue;
+  }
+  if (a.epi == EPI_SWIGLU) {
+    if (a.M % 128 != 0) {
+      snprintf(eb, el, "gemm: SwiGLU needs 2*d_ffn %% 128 == 0 (M=%d)", a.M);
+      return cudaErrorInvalidValue;
+    }
+    kp.m_tiles = a.M / 128;
+    kp.up_row0 = a.M / 2;
+  } else {
+    kp.m_tiles = (a.M + BM - 1) / BM;
+    kp.up_row0 = 0;
+  }
+  kp.kb = a.K / BK;
+  const long long tiles = (long long)kp.m_tiles * kp.n_tiles;
+  if (tiles > s.max_tiles) {
+    snprintf(eb, el, "gemm: %lld tiles exceed the counter table (%d)", tiles, s.max_tiles);
+    return cudaErrorInvalidValue;
+  }
+  kp.U = tiles * kp.kb;
+  kp.G = (int)((long long)grid < kp.U ? grid : kp.U);
+  if (s.ws_bytes < gemm_ws_bytes(kp.G)) {
+    snprintf(eb, el, "gemm: workspace too small");
+    return cudaErrorInvalidValue;
+  }
+  kp.ws = s.ws;
+  kp.counters = s.counters;
+  kp.err = s.err;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, a.W, a.K, a.M, 64, eb, el)) return cudaErrorInvalidValue;
+  if (!make_map(&mb, a.X, a.K, a.X_rows, BN, eb, el)) return cudaErrorInvalidValue;
+  return BN == 128 ? launch_bn<128>(a.epi, ma, mb, kp, stream, pdl) : launch_bn<256>(a.epi, ma, mb, kp, stream, pdl);
+}
+
+}  // namespace atspeed

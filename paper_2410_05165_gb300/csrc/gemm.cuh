@@ -1,0 +1,57 @@
+// Host-visible declarations of the weight-streaming GEMM (tcgen05 + TMA + TMEM).
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace atspeed {
+
+enum EpiKind : int { EPI_F32 = 0, EPI_BF16 = 1, EPI_RESID = 2, EPI_SWIGLU = 3, EPI_QKV = 4 };
+
+// Y[t][m] = sum_k W[m][k] * X[t][k]  (W: weight rows, X: token rows, both bf16 K-major)
+// with a fused epilogue.  The MMA runs "swap-AB": weight rows are the MMA M dimension (128 per
+// tile), tokens are the MMA N dimension (128 or 256 per tile), so a handful of tokens still
+// fills the tensor core while the weights stream from HBM exactly once.
+struct GemmArgs {
+  EpiKind epi;
+  const __nv_bfloat16* W;   // [M_rows][K]
+  const __nv_bfloat16* X;   // [X_rows][K], X_rows >= round_up(T, BN) (rows >= T are ignored)
+  int M;                    // weight rows (for EPI_SWIGLU: 2 * d_ffn, gate rows then up rows)
+  int K;                    // reduction length, multiple of 64
+  int T;                    // tokens
+  int X_rows;               // allocated token rows of X
+  // outputs
+  float* out_f32;           // EPI_F32 / EPI_RESID: [T][ldo]
+  __nv_bfloat16* out_bf16;  // EPI_BF16 / EPI_SWIGLU: [T][ldo]
+  int ldo;
+  // EPI_QKV
+  int d_model, head_dim;
+  const int* pos;           // [T] rotary positions
+  const int* kv_row;        // [T] destination row of k / v in the caches
+  const float* rope_cos;    // [max_pos][head_dim / 2]
+  const float* rope_sin;
+  __nv_bfloat16* q_out;     // [T][d_model]
+  __nv_bfloat16* k_cache;   // [rows][d_model]
+  __nv_bfloat16* v_cache;
+};
+
+struct GemmScratch {
+  float* ws;                // split partials: [2 * grid][256][128] fp32
+  int* counters;            // [max tiles], zero-initialised, restored to zero by every launch
+  size_t ws_bytes;
+  int max_tiles;
+  unsigned int* err;        // device error word
+};
+
+// Bytes of split-K workspace / counters needed for a grid of `grid` CTAs.
+size_t gemm_ws_bytes(int grid);
+int gemm_max_tiles();
+// Number of CTAs of the persistent stream-K grid (one per SM).
+int gemm_grid_size(int device);
+
+// Encodes the tensor maps and launches.  `pdl` enables programmatic dependent launch.
+cudaError_t gemm_launch(const GemmArgs& a, const GemmScratch& s, int grid, cudaStream_t stream, bool pdl,
+                        char* errbuf, size_t errlen);
+
+}  // namespace atspeed

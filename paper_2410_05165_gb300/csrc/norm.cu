@@ -1,0 +1,63 @@
+// Embedding gather and RMSNorm (LLaMA pre-norm), one CTA per token row.
+//   h[t] = embed[token[t]]                      (fp32 residual stream; the table is bf16)
+//   x[t] = bf16( h[t] / sqrt(mean(h[t]^2) + eps) * g )
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace atspeed {
+
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ h, const int* __restrict__ tokens,
+                                                      const __nv_bfloat16* __restrict__ embed,
+                                                      float* __restrict__ h_out, const __nv_bfloat16* __restrict__ g,
+                                                      int d, float eps, __nv_bfloat16* __restrict__ x, int ldx) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int t = blockIdx.x;
+  __shared__ float red[8];
+  float ss = 0.f;
+  if (tokens) {
+    const __nv_bfloat16* er = embed + (size_t)tokens[t] * d;
+    for (int i = threadIdx.x; i < d; i += blockDim.x) {
+      const float v = __bfloat162float(er[i]);
+      h_out[(size_t)t * d + i] = v;
+      ss += v * v;
+    }
+  } else {
+    const float* hr = h + (size_t)t * d;
+    for (int i = threadIdx.x; i < d; i += blockDim.x) {
+      const float v = hr[i];
+      ss += v * v;
+    }
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+    v = warp_sum(v);
+    if (threadIdx.x == 0) red[0] = v;
+  }
+  __syncthreads();
+  const float r = 1.0f / sqrtf(red[0] / (float)d + eps);
+  const float* hr = tokens ? h_out + (size_t)t * d : h + (size_t)t * d;
+  for (int i = threadIdx.x; i < d; i += blockDim.x)
+    x[(size_t)t * ldx + i] = __float2bfloat16_rn(hr[i] * r * __bfloat162float(g[i]));
+}
+
+cudaError_t rmsnorm_launch(const float* h, const int* tokens, const __nv_bfloat16* embed, float* h_out,
+                           const __nv_bfloat16* g, int T, int d, float eps, __nv_bfloat16* x, int ldx,
+                           cudaStream_t st, bool pdl) {
+  if (T <= 0) return cudaSuccess;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(T);
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  cfg.attrs = at;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, rmsnorm_kernel, h, tokens, embed, h_out, g, d, eps, x, ldx);
+}
+
+}  // namespace atspeed
