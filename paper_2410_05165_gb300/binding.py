@@ -23,7 +23,8 @@ PLAIN_TOPK, PLAIN_SAMPLE, SD_STRICT, SD_RELAXED = 0, 1, 2, 3
 
 EXPORTS = [
     "atspeed_create", "atspeed_destroy", "atspeed_last_error", "atspeed_prefill", "atspeed_begin_step",
-    "atspeed_draft_step", "atspeed_verify", "atspeed_beam_search", "atspeed_tree_shape", "atspeed_debug_tree",
+    "atspeed_draft_step", "atspeed_verify", "atspeed_draft_step_logits", "atspeed_verify_logits",
+    "atspeed_beam_search", "atspeed_tree_shape", "atspeed_debug_tree",
     "atspeed_debug_node_logits", "atspeed_set_tree", "atspeed_op_workspace_bytes", "atspeed_op_gemm",
     "atspeed_op_gemm_swiglu", "atspeed_op_rmsnorm", "atspeed_op_attention_scratch", "atspeed_op_attention",
 ]
@@ -82,6 +83,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "atspeed_begin_step": (c_int, [vp, vp, ctypes.POINTER(DecodeOpts)]),
         "atspeed_draft_step": (c_int, [vp, vp, ctypes.POINTER(DecodeOpts), c_int]),
         "atspeed_verify": (c_int, [vp, vp, ctypes.POINTER(DecodeOpts), c_int, vp, vp, vp, vp]),
+        "atspeed_draft_step_logits": (c_int, [vp, vp, ctypes.POINTER(DecodeOpts), c_int, fp]),
+        "atspeed_verify_logits": (c_int, [vp, vp, ctypes.POINTER(DecodeOpts), c_int, fp, vp, vp, vp, vp]),
         "atspeed_beam_search": (c_int, [vp, vp, c_int, vp, i32p, ctypes.POINTER(DecodeOpts), c_int, vp, vp, i32p]),
         "atspeed_tree_shape": (c_int, [vp, i32p, i32p, i32p, i32p]),
         "atspeed_debug_tree": (c_int, [vp, i32p, fp, fp, i32p]),
@@ -205,6 +208,26 @@ class Context:
         scores = torch.empty(B, K, dtype=torch.float32, device=dev)
         _check(self._lib.atspeed_verify(self.ptr, _stream(stream), ctypes.byref(o), mode, acc.data_ptr(),
                                         depth.data_ptr(), beams.data_ptr(), scores.data_ptr()), self.ptr)
+        return acc, depth, beams, scores
+
+    def draft_step_logits(self, o: DecodeOpts, mode: int, logits: np.ndarray, stream=None):
+        """logits [n_users][width][1024]: draft item-code logits of the previous level's slots."""
+        lg = np.ascontiguousarray(logits, np.float32)
+        _check(self._lib.atspeed_draft_step_logits(self.ptr, _stream(stream), ctypes.byref(o), mode,
+                                                   lg.ctypes.data_as(ctypes.POINTER(ctypes.c_float))), self.ptr)
+
+    def verify_logits(self, o: DecodeOpts, mode: int, logits: np.ndarray, stream=None):
+        """logits [n_users][K + gamma*N][1024]: target item-code logits of every node slot."""
+        B, K = self.n_users, o.K
+        dev = torch.device("cuda")
+        acc = torch.empty(B, dtype=torch.int32, device=dev)
+        depth = torch.empty(B, dtype=torch.int32, device=dev)
+        beams = torch.empty(B, K, 4, dtype=torch.int32, device=dev)
+        scores = torch.empty(B, K, dtype=torch.float32, device=dev)
+        lg = np.ascontiguousarray(logits, np.float32)
+        _check(self._lib.atspeed_verify_logits(self.ptr, _stream(stream), ctypes.byref(o), mode,
+                                               lg.ctypes.data_as(ctypes.POINTER(ctypes.c_float)), acc.data_ptr(),
+                                               depth.data_ptr(), beams.data_ptr(), scores.data_ptr()), self.ptr)
         return acc, depth, beams, scores
 
     def beam_search(self, tokens: torch.Tensor, offsets: Sequence[int], o: DecodeOpts, mode: int, stream=None,

@@ -1135,11 +1135,6 @@ atspeed_status atspeed_beam_search(atspeed_ctx* c, atspeed_stream stream, int n_
       for (auto& us : c->users) any |= us.active;
       if (!any) break;
       open_step(c, &o, st);
-      if (!sd) {
-        // plain beam search: Philox counter word sd_step = 0 at every level
-        for (auto& us : c->users) us.step = 0;
-        upload_users(c, st);
-      }
       int maxg = 0;
       for (auto& us : c->users)
         if (us.active) maxg = std::max(maxg, us.g);

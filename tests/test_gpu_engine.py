@@ -1,0 +1,241 @@
+"""Call-level parity of the speculative verification engine against the oracle, through the C ABI.
+
+* Discrete logic (drafting, strict and relaxed verification, plain top-K and sampling beam search)
+  driven by the same seeded synthetic logits on both sides: bit-exact beams, accepted lengths and
+  scores over whole multi-step decodes, several users with their own Philox streams.
+* The bf16 decoder: tree-node logits of a seeded drafted tree (tree attention over the paged
+  prefix) against the oracle's per-path causal forward, within 2e-2.
+* End to end: speculative strict decoding returns exactly the plain target beam search (lossless,
+  bitwise on the GPU) and the oracle's ranked items (up to near-ties of the bf16 forward).
+"""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle.model import Model, PathEvaluator
+from oracle.sd import plain_beam_search, sd_decode
+from oracle.trie import Trie
+
+pytestmark = pytest.mark.gpu
+
+L = 4
+
+
+@pytest.fixture(scope="module")
+def ats():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2410_05165_gb300 as m
+    return m
+
+
+def hashed_row(seed, user, path, std=3.0):
+    return (np.random.default_rng([seed, user, len(path), *path]).standard_normal(256) * std).astype(np.float32)
+
+
+def rows_fn(seed, user, std=3.0):
+    return lambda paths: [hashed_row(seed, user, p, std) for p in paths]
+
+
+def _ctx(ats, spec_t, spec_d, items, code_base, B, P, K, N, G, seed=1):
+    tw = ats.weights_to_device(synth.model_weights(spec_t, seed, "target"))
+    dw = ats.weights_to_device(synth.model_weights(spec_d, seed, "draft")) if spec_d is not None else None
+    return ats.Context(spec_t, tw, spec_d, dw, items, code_base, max_users=B, max_prompt=P, max_K=K, max_N=N,
+                       max_gamma=G)
+
+
+def _prefill(ats, ctx, prompts):
+    toks = torch.from_numpy(np.concatenate(prompts).astype(np.int32)).cuda()
+    off = np.concatenate([[0], np.cumsum([len(p) for p in prompts])]).astype(np.int32)
+    ctx.prefill(toks, off)
+    return toks, off
+
+
+def _paths_of(tree, u):
+    return [tuple(int(c) for c in p if c >= 0) for p in tree["path"][u]]
+
+
+# ------------------------------------------------------------------------------------------------
+# discrete logic on synthetic logits
+# ------------------------------------------------------------------------------------------------
+
+def _drive_logits_decode(ats, ctx, B, K, N, G, mode, seed_t, seed_d, philox):
+    """Runs a whole speculative decode through draft_step_logits / verify_logits, feeding every
+    node the hashed logits of its path; returns per-user (paths, scores, steps)."""
+    o = ats.opts(K, N, G, philox)
+    steps = [[] for _ in range(B)]
+    fin = [None] * B
+    for it in range(2 * L):
+        ctx.begin_step(o)
+        tree = ctx.debug_tree(G)
+        depth = tree["depth"]
+        if np.all(depth >= L):
+            break
+        si, sl = tree["slots_in"], tree["slots_lvl"]
+        gmax = int(max(min(G, L - int(d)) for d in depth if d < L))
+        for j in range(1, gmax + 1):
+            tree = ctx.debug_tree(G)
+            width = si if j == 1 else sl
+            off = 0 if j == 1 else si + (j - 2) * sl
+            lg = np.zeros((B, width, 1024), np.float32)
+            for u in range(B):
+                paths = _paths_of(tree, u)
+                for k in range(width):
+                    p = paths[off + k]
+                    lg[u, k, 256 * len(p):256 * (len(p) + 1)] = hashed_row(seed_d, u, p)
+            ctx.draft_step_logits(o, mode, lg)
+        tree = ctx.debug_tree(G)
+        stride = si + G * sl
+        lt = np.zeros((B, stride, 1024), np.float32)
+        for u in range(B):
+            for k, p in enumerate(_paths_of(tree, u)):
+                if len(p) < L and (k < si or len(p) > 0):
+                    lt[u, k, 256 * len(p):256 * (len(p) + 1)] = hashed_row(seed_t, u, p)
+        acc, dep, beams, sc = ctx.verify_logits(o, mode, lt)
+        for u in range(B):
+            if depth[u] < L:
+                steps[u].append((int(depth[u]), int(acc[u])))
+        last_beams, last_sc, last_dep = beams.cpu().numpy(), sc.cpu().numpy(), dep.cpu().numpy()
+        for u in range(B):
+            if fin[u] is None and last_dep[u] >= L:
+                fin[u] = ([tuple(int(c) for c in r) for r in last_beams[u] if r[0] >= 0], last_sc[u])
+    return fin, steps
+
+
+@pytest.mark.parametrize("K,N,G,mode", [(5, 10, 2, 0), (10, 40, 4, 0), (3, 8, 3, 1), (10, 40, 4, 1), (20, 80, 4, 1),
+                                         (1, 1, 4, 0), (1, 1, 1, 1), (4, 4, 2, 1)])
+def test_decode_logic_bit_exact_on_synthetic_logits(ats, K, N, G, mode):
+    """Drafting, strict / relaxed verification and the commit of accepted beams, over whole decodes
+    of 3 users, against oracle.sd_decode on the same hashed logits: identical items, scores and
+    accepted lengths (no floating-point tolerance: both sides compute in fp32)."""
+    items = synth.make_items(4000, "zipf", 1.1, 11)
+    trie = Trie(items)
+    spec = synth.ModelSpec(1, 64, 2, 128, 1024)
+    B, philox = 3, 12345
+    ctx = _ctx(ats, spec, spec, items, 0, B, 16, K, N, G)
+    _prefill(ats, ctx, [np.arange(5 + u, dtype=np.int32) for u in range(B)])
+    fin, steps = _drive_logits_decode(ats, ctx, B, K, N, G, mode, 100, 200, philox)
+    for u in range(B):
+        ref, ref_sc, st = sd_decode(rows_fn(100, u), rows_fn(200, u), trie, K, N, G,
+                                    "relaxed" if mode == 1 else "strict", seed=philox, user=u)
+        got, got_sc = fin[u]
+        assert got == ref, (u, got, ref)
+        np.testing.assert_array_equal(got_sc[:len(ref)], ref_sc)
+        assert [a for (_, a) in steps[u]] == [s[1] for s in st.steps]
+        assert [d for (d, _) in steps[u]] == [s[0] for s in st.steps]
+    ctx.close()
+
+
+@pytest.mark.parametrize("sample", [False, True])
+def test_plain_beam_search_logic_on_synthetic_logits(ats, sample):
+    """gamma = 0: plain top-K beam search (strict) / sampling beam search (relaxed)."""
+    items = synth.make_items(3000, "uniform", 1.1, 12)
+    trie = Trie(items)
+    spec = synth.ModelSpec(1, 64, 2, 128, 1024)
+    B, K = 2, 6
+    ctx = _ctx(ats, spec, None, items, 0, B, 8, K, 1, 1)
+    _prefill(ats, ctx, [np.arange(4, dtype=np.int32)] * B)
+    o = ats.opts(K, 1, 0, 77)
+    for lvl in range(L):
+        ctx.begin_step(o)
+        tree = ctx.debug_tree(0)
+        si = tree["slots_in"]
+        lt = np.zeros((B, si, 1024), np.float32)
+        for u in range(B):
+            for k, p in enumerate(_paths_of(tree, u)[:si]):
+                lt[u, k, 256 * len(p):256 * (len(p) + 1)] = hashed_row(300, u, p)
+        _, _, beams, sc = ctx.verify_logits(o, 1 if sample else 0, lt)
+    for u in range(B):
+        ref, ref_sc = plain_beam_search(rows_fn(300, u), trie, K, sample=sample, seed=77, user=u)
+        got = [tuple(int(c) for c in r) for r in beams[u].cpu().numpy()]
+        assert got == ref
+        np.testing.assert_array_equal(sc[u].cpu().numpy(), ref_sc)
+    ctx.close()
+
+
+# ------------------------------------------------------------------------------------------------
+# the bf16 decoder
+# ------------------------------------------------------------------------------------------------
+
+def _tree_arrays(levels, B, n_levels, width):
+    cnt = np.zeros((B, n_levels), np.int32)
+    par = np.zeros((B, n_levels, width), np.int32)
+    cod = np.zeros((B, n_levels, width), np.int32)
+    sq = np.zeros((B, n_levels, width), np.float32)
+    for j, lvl in enumerate(levels):
+        cnt[0, j] = len(lvl)
+        for k, (p, c) in enumerate(lvl):
+            par[0, j, k] = p
+            cod[0, j, k] = c
+            sq[0, j, k] = -float(k)
+    return cnt, par, cod, sq
+
+
+@pytest.mark.parametrize("cfg,layers", [("tiny", None), ("mid", 2), ("7b", 1)])
+def test_tree_node_logits_match_oracle(ats, cfg, layers):
+    """Target item-code logits of every node of a seeded drafted tree (levels 1..3, the
+    verification call's forward with tree attention over the paged prefix) and of the prefill's
+    last position, against the oracle's causal forward of prompt + path."""
+    w = synth.workload(cfg)
+    spec = w.target if layers is None else synth.ModelSpec(layers, w.target.d_model, w.target.n_heads,
+                                                          w.target.d_ffn, w.target.vocab)
+    items = synth.make_items(min(w.n_items, 5000), w.code_dist, w.zipf_a, w.seed)
+    prompt = synth.make_prompts(1, w.prompt_len, spec.vocab, w.seed)[0]
+    K, N, G = w.K, w.N, 3
+    ctx = _ctx(ats, spec, None, items, w.code_base, 1, len(prompt), K, N, G, seed=w.seed)
+    _prefill(ats, ctx, [prompt])
+    incoming, levels = synth.random_tree(items, 0, 1, G, N, seed=5)
+    o = ats.opts(K, N, G)
+    ctx.begin_step(o)
+    cnt, par, cod, sq = _tree_arrays(levels, 1, G, N)
+    ctx.set_tree(cnt, par, cod, sq)
+    root = ctx.node_logits(0, 0, 0)
+    ctx.verify(o, ats.STRICT)
+    tw = synth.model_weights(spec, w.seed, "target")
+    ev = PathEvaluator(Model(spec, tw, w.code_base), prompt)
+    np.testing.assert_allclose(root, ev.root_logits, atol=2e-2)
+    paths = [()]
+    off = K
+    worst = 0.0
+    prev = [()]
+    for j, lvl in enumerate(levels):
+        cur = [prev[p] + (c,) for p, c in lvl]
+        ref = ev.logits(cur)
+        for k, p in enumerate(cur):
+            got = ctx.node_logits(0, 0, off + k)
+            worst = max(worst, float(np.abs(got - ref[k]).max()))
+        off += N
+        prev = cur
+    assert worst < 2e-2, worst
+    ctx.close()
+
+
+def test_sd_strict_lossless_and_matches_oracle_tiny(ats):
+    """Tiny workload end to end: SD strict == plain target beam search bitwise on the GPU, and
+    equal to the oracle's plain beam search up to near-ties of the bf16 forward."""
+    w = synth.workload("tiny")
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    prompts = synth.make_prompts(2, w.prompt_len, w.target.vocab, w.seed)
+    ctx = _ctx(ats, w.target, w.draft, items, w.code_base, 2, 32, w.K, w.N, w.gamma, seed=w.seed)
+    toks = torch.from_numpy(np.concatenate(prompts)).cuda()
+    off = [0, len(prompts[0]), len(prompts[0]) + len(prompts[1])]
+    o = ats.opts(w.K, w.N, w.gamma)
+    sd_items, sd_sc, stats = ctx.beam_search(toks, off, o, ats.SD_STRICT)
+    pl_items, pl_sc, _ = ctx.beam_search(toks, off, o, ats.PLAIN_TOPK)
+    np.testing.assert_array_equal(sd_items.cpu().numpy(), pl_items.cpu().numpy())
+    np.testing.assert_array_equal(sd_sc.cpu().numpy(), pl_sc.cpu().numpy())
+    assert np.all(stats[:, 1] >= 1)
+    tw = synth.model_weights(w.target, w.seed, "target")
+    trie = Trie(items)
+    for u in range(2):
+        ev = PathEvaluator(Model(w.target, tw, w.code_base), prompts[u])
+        ref, ref_sc = plain_beam_search(
+            lambda ps: [ev.logits([p])[0][256 * len(p):256 * (len(p) + 1)].astype(np.float32) for p in ps],
+            trie, w.K)
+        got = [tuple(int(c) for c in r) for r in sd_items[u].cpu().numpy()]
+        np.testing.assert_allclose(sd_sc[u].cpu().numpy(), ref_sc, atol=2e-2)
+        if got != ref:
+            gaps = np.abs(np.diff(ref_sc.astype(np.float64)))
+            assert gaps.min() < 2e-2, (got, ref)
+    ctx.close()
