@@ -1,0 +1,328 @@
+#!/usr/bin/env python3
+"""Throughput of speculative beam decoding with strict top-K verification on the 7B-shape workload.
+
+One step = one recommendation list per user: prefill of the user history, then speculative steps
+(gamma = 4 drafted beam-search steps of width N = 40 by the draft model, one verification call of
+the 7B-shape target over the whole drafted tree, strict top-K verification with K = 10) until every
+user holds K complete items.  Metric: rec lists/s (whole job), with the verification call's HBM
+roofline fraction and the weight-streaming GEMM's achieved bandwidth measured live.
+
+Weights are seeded random-init of the LLaMA-7B shape (the paper's trained LC-Rec / LLaMA-68M
+weights and datasets are not available); inputs are synthetic (see synth/world.py).  Inputs are
+larger than L2: every step streams the 13.5 GB of target weights several times.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload 7b]
+                  [--mode strict|relaxed]
+Under torchrun every rank decodes its own users (replicas, no collective on the data path).
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "rec lists/sec (7B-shape target, K=10); verify-call % of HBM roofline"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="7b")
+    ap.add_argument("--mode", choices=["strict", "relaxed"], default="strict")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+def verify_bytes_flops(w, T, P_users):
+    """Algorithmic bytes / FLOPs of one verification call: weights once, item-code LM-head rows,
+    every user's prefix KV read once, the tree's node KV written (bf16)."""
+    t = w.target
+    d, f, Lr = t.d_model, t.d_ffn, t.n_layers
+    per_layer = 4 * d * d + 3 * d * f
+    B = 2 * Lr * per_layer + 2 * 1024 * d + sum(P_users) * Lr * 2 * d * 2 + T * Lr * 2 * d * 2
+    F = 2 * T * Lr * per_layer + sum(4 * (T / len(P_users)) * (P + 2) * d * Lr for P in P_users) + 2 * T * d * 1024
+    return B, F
+
+
+# ----------------------------------------------------------------------------------------------
+# CPU oracle leg (bounded sample)
+# ----------------------------------------------------------------------------------------------
+
+def oracle_sample(w, mode, layers=1):
+    """One recommendation list of the oracle with the target truncated to `layers` of its layers and
+    the draft to one layer; returns (seconds for the sample, seconds scaled to the full model)."""
+    from oracle.model import Model, PathEvaluator
+    from oracle.sd import sd_decode
+    from oracle.trie import Trie
+    tspec = synth.ModelSpec(layers, w.target.d_model, w.target.n_heads, w.target.d_ffn, w.target.vocab)
+    dspec = synth.ModelSpec(1, w.draft.d_model, w.draft.n_heads, w.draft.d_ffn, w.draft.vocab)
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    prompt = synth.make_prompts(1, w.prompt_len, w.target.vocab, w.seed)[0]
+    tm = Model(tspec, synth.model_weights(tspec, w.seed, "target"), w.code_base)
+    dm = Model(dspec, synth.model_weights(dspec, w.seed, "draft"), w.code_base)
+    trie = Trie(items)
+    t0 = time.perf_counter()
+    te, de = PathEvaluator(tm, prompt), PathEvaluator(dm, prompt)
+
+    def rows(ev):
+        return lambda ps: [r[256 * len(p):256 * (len(p) + 1)].astype(np.float32) for p, r in zip(ps, ev.logits(ps))]
+    sd_decode(rows(te), rows(de), trie, w.K, w.N, w.gamma, mode, seed=w.philox_seed)
+    dt = time.perf_counter() - t0
+    return dt, dt * w.target.n_layers / layers
+
+
+def run_reference(args, w):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    cores = os.cpu_count()
+    times = []
+    for i in range(args.warmup + args.steps):
+        _, scaled = oracle_sample(w, args.mode)
+        if i >= args.warmup:
+            times.append(scaled)
+    per_list = statistics.mean(times)
+    value = 1.0 / per_list
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "rec lists/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_list * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{w.name}: 7B-shape target, 4-layer d=768 draft, K={w.K}, N={w.N}, gamma={w.gamma}, "
+                               f"P={w.prompt_len[0]}, {w.n_items} items, {args.mode} verification, batch 1"},
+        "cpu_baseline": {"value": value, "unit": "rec lists/s", "cores": cores, "kind": "oracle",
+                         "sample": "one rec list with the target cut to 1 of 32 layers and the draft to 1 layer, "
+                                   "time x32"},
+        "e2e": {"value": value, "unit": "rec lists/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------------------------
+# GPU leg
+# ----------------------------------------------------------------------------------------------
+
+class Clocks:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu):
+        self.gpu = gpu
+        self.p = None
+        self.f = tempfile.NamedTemporaryFile(mode="w+", suffix=".csv", delete=False)
+
+    def start(self):
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                       "-lms", "100", "-i", str(self.gpu)], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.p.terminate()
+        self.p.wait()
+        self.f.flush()
+        self.f.seek(0)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.f.read().splitlines():
+            t = [x.strip() for x in line.split(",")]
+            if len(t) < 9:
+                continue
+            try:
+                sm.append(float(t[1]))
+                mx.append(float(t[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, t[5:9]):
+                if v.lower() in ("active", "0x1", "1"):
+                    reasons.add(n)
+        os.unlink(self.f.name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def run_ours(args, w):
+    import torch
+    import torch.distributed as dist
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+    import paper_2410_05165_gb300 as ats
+    try:
+        ats.load()
+    except RuntimeError:
+        from paper_2410_05165_gb300.build import build
+        build()
+        ats.load()
+    mode = ats.SD_STRICT if args.mode == "strict" else ats.SD_RELAXED
+    vmode = ats.STRICT if args.mode == "strict" else ats.RELAXED
+
+    def to_dev(spec, role):
+        out = {}
+        for name, arr in synth.iter_model_tensors(spec, w.seed, role):
+            out[name] = torch.from_numpy(arr).to(device="cuda", dtype=torch.bfloat16)
+        return out
+    tw, dw = to_dev(w.target, "target"), to_dev(w.draft, "draft")
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    prompts = synth.make_prompts(w.n_users * world, w.prompt_len, w.target.vocab, w.seed)[
+        rank * w.n_users:(rank + 1) * w.n_users]
+    B = len(prompts)
+    P_users = [len(p) for p in prompts]
+    ctx = ats.Context(w.target, tw, w.draft, dw, items, w.code_base, max_users=B, max_prompt=max(P_users),
+                      max_K=w.K, max_N=w.N, max_gamma=w.gamma)
+    h_tok = torch.from_numpy(np.concatenate(prompts).astype(np.int32)).pin_memory()
+    toks = h_tok.cuda()
+    offsets = np.concatenate([[0], np.cumsum(P_users)]).astype(np.int32)
+    o = ats.opts(w.K, w.N, w.gamma, w.philox_seed)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+
+    # ---- warm-up, then K timed steps (inputs resident in HBM)
+    for _ in range(args.warmup):
+        ctx.beam_search(toks, offsets, o, mode)
+    barrier()
+    clocks = Clocks(local)
+    clocks.start()
+    l0 = ctx.profile_read(-1)["launches"]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    stats = None
+    for _ in range(args.steps):
+        _, _, stats = ctx.beam_search(toks, offsets, o, mode)
+    e1.record(stream)
+    barrier()
+    clk = clocks.stop()
+    launches = (ctx.profile_read(-1)["launches"] - l0) / args.steps
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = B * world * args.steps / (ms / 1e3)
+
+    # ---- end to end through the C ABI: pinned host prompt -> device, decode, items -> host
+    h_items = torch.empty(B, w.K, 4, dtype=torch.int32).pin_memory()
+    h_sc = torch.empty(B, w.K, dtype=torch.float32).pin_memory()
+    d_items = torch.empty(B, w.K, 4, dtype=torch.int32, device="cuda")
+    d_sc = torch.empty(B, w.K, dtype=torch.float32, device="cuda")
+    barrier()
+    e0.record(stream)
+    for _ in range(args.steps):
+        toks.copy_(h_tok, non_blocking=True)
+        ctx.beam_search(toks, offsets, o, mode, items_out=d_items, scores_out=d_sc)
+        h_items.copy_(d_items, non_blocking=True)
+        h_sc.copy_(d_sc, non_blocking=True)
+    e1.record(stream)
+    barrier()
+    ms_e2e = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms_e2e], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_e2e = float(t.item())
+    e2e = {"value": B * world * args.steps / (ms_e2e / 1e3), "unit": "rec lists/s",
+           "h2d_bytes_per_step": int(h_tok.numel() * 4), "d2h_bytes_per_step": int(h_items.numel() * 4 + h_sc.numel() * 4)}
+
+    # ---- the verification call alone (first call of a decode: depth 0, T = 3 N tree tokens)
+    hbm, tf, peak_kind = peaks()
+    ver_ms, gemm = [], {"ms": 0.0, "bytes": 0.0, "launches": 0, "flops": 0.0}
+    for rep in range(3 + args.steps):
+        ctx.prefill(toks, offsets)
+        ctx.begin_step(o)
+        for _ in range(w.gamma):
+            ctx.draft_step(o, vmode)
+        prof = rep >= 3 + args.steps - 2
+        if prof:
+            ctx.profile(True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        ctx.verify(o, vmode)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if prof:
+            for k in range(4):
+                r = ctx.profile_read(k)
+                for key in gemm:
+                    gemm[key] += r[key]
+            ctx.profile(False)
+        elif rep >= 3:
+            ver_ms.append(e0.elapsed_time(e1))
+    T_first = min(w.gamma, 3) * w.N * B
+    vb, vf = verify_bytes_flops(w, T_first, P_users)
+    v_ms = statistics.median(ver_ms)
+    t_roof = max(vb / (hbm * 1e9), vf / (tf * 1e12)) * 1e3
+    g_gbs = gemm["bytes"] / (gemm["ms"] / 1e3) / 1e9
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "rec lists/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights, synthetic items)",
+        "config": {"workload": f"{w.name}: 7B-shape target (32L d4096 H32 ffn11008 V33024), draft 4L d768, "
+                               f"K={w.K} N={w.N} gamma={w.gamma}, P={w.prompt_len[0]}, {w.n_items} Zipf items, "
+                               f"{args.mode} verification, {B} user(s) per GPU",
+                   "l2": "inputs larger than L2 (13.5 GB of target weights per verification call)"},
+        "roofline": {"bound": "hbm", "achieved": g_gbs, "peak": hbm, "unit": "GB/s", "frac": g_gbs / hbm,
+                     "traffic": None, "kernel": "gemm_kernel (tcgen05 weight-streaming GEMM) in the verification call",
+                     "peak_source": peak_kind, "launches": gemm["launches"],
+                     "avg_launch_us": gemm["ms"] / max(1, gemm["launches"]) * 1e3},
+        "verify_call": {"ms": v_ms, "tree_tokens": T_first, "alg_bytes": vb, "alg_flops": vf,
+                        "t_roof_ms": t_roof, "frac_of_roofline": t_roof / v_ms, "peak_source": peak_kind},
+        "accepted_steps_per_list": float(np.mean(stats[:, 0])), "verify_calls_per_list": float(np.mean(stats[:, 1])),
+        "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
+    }
+    if rank == 0 and world == 1:
+        cores = os.cpu_count()
+        samp, scaled = oracle_sample(w, args.mode)
+        line["cpu_baseline"] = {"value": 1.0 / scaled, "unit": "rec lists/s", "cores": cores, "kind": "oracle",
+                                "sample": f"one rec list with the target cut to 1 of 32 layers (draft 1 layer), "
+                                          f"{samp:.1f} s, time x32"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    ctx.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    w = synth.workload(args.workload)
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_ours(args, w)
+
+
+if __name__ == "__main__":
+    main()

@@ -165,6 +165,17 @@ atspeed_status atspeed_beam_search(atspeed_ctx *ctx, atspeed_stream stream, int 
  * Introspection / test hooks.
  * ---------------------------------------------------------------------------------------------- */
 
+/* Per-launch timing: while enabled, every kernel launch of the decoder forwards is bracketed by
+ * CUDA events on its stream (and programmatic dependent launch is off, so launches do not
+ * overlap).  atspeed_profile(ctx, 1) clears previous records.  profile_read sums, over the
+ * launches of one kind (0 QKV GEMM, 1 O GEMM, 2 gate/up GEMM, 3 down GEMM, 4 LM-head GEMM,
+ * 5 attention), the launch count, the device time (ms), and the algorithmic bytes and FLOPs (weights
+ * read once, activations in, outputs out).  kind < 0 returns in *h_launches the number of kernels
+ * the context has launched since creation (every kind, profiling on or off).  Synchronises. */
+atspeed_status atspeed_profile(atspeed_ctx *ctx, int enable);
+atspeed_status atspeed_profile_read(atspeed_ctx *ctx, int kind, int32_t *h_launches, double *h_ms, double *h_bytes,
+                                    double *h_flops);
+
 /* Shape of the current speculative step: h_depth[n_users], h_levels[n_users] (drafted levels),
  * and the node-table geometry (*h_slots_in slots on level 0, *h_slots_lvl per drafted level). */
 atspeed_status atspeed_tree_shape(const atspeed_ctx *ctx, int32_t *h_depth, int32_t *h_levels, int32_t *h_slots_in,
@@ -213,7 +224,9 @@ atspeed_status atspeed_op_rmsnorm(atspeed_stream stream, const float *d_h, const
                                   void *d_x, int ldx);
 
 /* Tree attention of T query tokens of ONE user over a paged prefix of length P plus per-token path
- * keys (Sec. 3.3, App. A.3.1).  q bf16 [T][H*hd]; caches bf16 [rows][H*hd]; prefix row p of the
+ * keys (Sec. 3.3, App. A.3.1).  q bf16 [T][H*hd]; K cache bf16 [rows][H*hd]; V cache fp16
+ * [rows][H*hd] holding bf16-rounded values (the library's own layout: P V runs in fp16 with P split
+ * into two fp16 halves); prefix row p of the
  * user is cache row 64*h_pages[p/64] + p%64; token t also attends to the n_path[t] <= 4 cache rows
  * path_rows[t][0..], and sees prefix positions < vis[t] (vis[t] = P for tree nodes, t+1 for a
  * causal prefill).  out bf16 [T][H*hd].  d_part: fp32 scratch of atspeed_op_attention_scratch(T,H,hd,P). */

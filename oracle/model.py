@@ -145,10 +145,18 @@ class PathEvaluator:
         self.cache: Dict[Tuple[int, ...], Tuple[list, np.ndarray]] = {}
 
     def logits(self, paths: Sequence[Tuple[int, ...]]) -> List[np.ndarray]:
-        """fp64 logit rows (item-code rows, or the whole vocabulary) at the end of each path."""
-        want = sorted({tuple(p) for p in paths}, key=len)
-        for p in want:
-            self._ensure(p)
+        """fp64 logit rows (item-code rows, or the whole vocabulary) at the end of each path.
+
+        Missing paths (and their missing ancestors) are computed one depth at a time, all paths of
+        a depth together, so each weight matrix is read once per depth."""
+        missing = set()
+        for p in paths:
+            p = tuple(p)
+            while len(p) > 0 and p not in self.cache and p not in missing:
+                missing.add(p)
+                p = p[:-1]
+        for t in sorted({len(p) for p in missing}):
+            self._extend(sorted(p for p in missing if len(p) == t))
         return [self.root_logits if len(p) == 0 else self.cache[tuple(p)][1] for p in paths]
 
     def _ensure(self, path: Tuple[int, ...]) -> None:

@@ -24,7 +24,7 @@ PLAIN_TOPK, PLAIN_SAMPLE, SD_STRICT, SD_RELAXED = 0, 1, 2, 3
 EXPORTS = [
     "atspeed_create", "atspeed_destroy", "atspeed_last_error", "atspeed_prefill", "atspeed_begin_step",
     "atspeed_draft_step", "atspeed_verify", "atspeed_draft_step_logits", "atspeed_verify_logits",
-    "atspeed_beam_search", "atspeed_tree_shape", "atspeed_debug_tree",
+    "atspeed_beam_search", "atspeed_profile", "atspeed_profile_read", "atspeed_tree_shape", "atspeed_debug_tree",
     "atspeed_debug_node_logits", "atspeed_set_tree", "atspeed_op_workspace_bytes", "atspeed_op_gemm",
     "atspeed_op_gemm_swiglu", "atspeed_op_rmsnorm", "atspeed_op_attention_scratch", "atspeed_op_attention",
 ]
@@ -86,6 +86,9 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "atspeed_draft_step_logits": (c_int, [vp, vp, ctypes.POINTER(DecodeOpts), c_int, fp]),
         "atspeed_verify_logits": (c_int, [vp, vp, ctypes.POINTER(DecodeOpts), c_int, fp, vp, vp, vp, vp]),
         "atspeed_beam_search": (c_int, [vp, vp, c_int, vp, i32p, ctypes.POINTER(DecodeOpts), c_int, vp, vp, i32p]),
+        "atspeed_profile": (c_int, [vp, c_int]),
+        "atspeed_profile_read": (c_int, [vp, c_int, i32p, ctypes.POINTER(ctypes.c_double),
+                                         ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]),
         "atspeed_tree_shape": (c_int, [vp, i32p, i32p, i32p, i32p]),
         "atspeed_debug_tree": (c_int, [vp, i32p, fp, fp, i32p]),
         "atspeed_debug_node_logits": (c_int, [vp, c_int, c_int, c_int, fp]),
@@ -243,6 +246,16 @@ class Context:
                                              mode, items.data_ptr(), scores.data_ptr(),
                                              stats.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))), self.ptr)
         return items, scores, stats
+
+    def profile(self, enable: bool):
+        _check(self._lib.atspeed_profile(self.ptr, 1 if enable else 0), self.ptr)
+
+    def profile_read(self, kind: int):
+        n = ctypes.c_int32()
+        ms, by, fl = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+        _check(self._lib.atspeed_profile_read(self.ptr, kind, ctypes.byref(n), ctypes.byref(ms), ctypes.byref(by),
+                                              ctypes.byref(fl)), self.ptr)
+        return {"launches": n.value, "ms": ms.value, "bytes": by.value, "flops": fl.value}
 
     # -- introspection -----------------------------------------------------------------------------
     def tree_shape(self):

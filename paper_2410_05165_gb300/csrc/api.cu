@@ -40,7 +40,8 @@ struct ModelRt {
   const bf16 *embed = nullptr, *final_norm = nullptr, *lm_head = nullptr;
   std::vector<const bf16*> attn_norm, wqkv, wo, mlp_norm, wgate_up, wdown;
   // KV arena: [layers][rows][d]
-  bf16 *kc = nullptr, *vc = nullptr;
+  bf16* kc = nullptr;
+  __half* vc = nullptr;
   int rows = 0;
   std::vector<CUtensorMap> mk, mv;
   float *rope_cos = nullptr, *rope_sin = nullptr;  // [max_pos][hd/2]
@@ -115,6 +116,16 @@ struct atspeed_ctx {
   std::vector<UserState> users;
   std::vector<void*> allocs;
   bool pdl = true;
+  // optional per-launch timing (CUDA events on the launching stream)
+  bool prof = false;
+  struct ProfRec {
+    int kind;
+    double bytes, flops;
+    cudaEvent_t a, b;
+  };
+  std::vector<ProfRec> prof_recs;
+  std::vector<cudaEvent_t> prof_pool;
+  long long n_launch = 0;  // kernels launched by this context (all kinds)
 };
 
 namespace {
@@ -228,7 +239,7 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.rows = L.max_users * (c->prefix_pages_per_user * ATT_PAGE + c->node_rows_per_user);
   const size_t per = (size_t)m.rows * m.d;
   m.kc = dalloc<bf16>(c, per * m.layers);
-  m.vc = dalloc<bf16>(c, per * m.layers);
+  m.vc = dalloc<__half>(c, per * m.layers);
   m.mk.resize(m.layers);
   m.mv.resize(m.layers);
   char eb[256];
@@ -391,13 +402,51 @@ struct FwdPlan {
   int logit_row_base = 0;
 };
 
-void gemm(atspeed_ctx* c, const GemmArgs& a, cudaStream_t st) {
+cudaEvent_t prof_event(atspeed_ctx* c) {
+  if (!c->prof_pool.empty()) {
+    cudaEvent_t e = c->prof_pool.back();
+    c->prof_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e;
+  CK(cudaEventCreate(&e));
+  return e;
+}
+
+// Brackets one kernel launch with events when profiling is on.
+struct ProfScope {
+  atspeed_ctx* c;
+  cudaStream_t st;
+  atspeed_ctx::ProfRec r;
+  ProfScope(atspeed_ctx* c_, cudaStream_t st_, int kind, double bytes, double flops) : c(c_), st(st_) {
+    if (!c->prof) return;
+    r.kind = kind;
+    r.bytes = bytes;
+    r.flops = flops;
+    r.a = prof_event(c);
+    r.b = prof_event(c);
+    CK(cudaEventRecord(r.a, st));
+  }
+  void done() {
+    if (!c->prof) return;
+    CK(cudaEventRecord(r.b, st));
+    c->prof_recs.push_back(r);
+  }
+};
+
+void gemm(atspeed_ctx* c, const GemmArgs& a, cudaStream_t st, int kind) {
   char eb[256] = {0};
-  cudaError_t e = gemm_launch(a, c->gs, c->gemm_grid, st, c->pdl, eb, sizeof eb);
+  // algorithmic bytes: weights once, activations in, outputs out
+  const double out_b = a.epi == EPI_F32 ? 4.0 * a.M : a.epi == EPI_RESID ? 8.0 * a.M
+                       : a.epi == EPI_SWIGLU ? 1.0 * a.M : 2.0 * a.M;
+  ProfScope ps(c, st, kind, 2.0 * a.M * a.K + 2.0 * a.T * a.K + out_b * a.T, 2.0 * a.M * a.K * a.T);
+  cudaError_t e = gemm_launch(a, c->gs, c->gemm_grid, st, c->pdl && !c->prof, eb, sizeof eb);
+  c->n_launch += 1;
   if (e != cudaSuccess) {
     set_err(c, "gemm launch failed: %s %s", cudaGetErrorString(e), eb);
     throw Fail{ATSPEED_E_CUDA};
   }
+  ps.done();
 }
 
 void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
@@ -420,6 +469,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
   for (int l = 0; l < m.layers; ++l) {
     CK(rmsnorm_launch(m.h, l == 0 ? p.d_tokens : nullptr, m.embed, m.h, m.attn_norm[l], T, m.d, m.eps, m.x, m.d, st,
                       pdl));
+    c->n_launch += 1;
     GemmArgs g = {};
     g.epi = EPI_QKV;
     g.W = m.wqkv[l];
@@ -437,7 +487,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.q_out = m.q;
     g.k_cache = m.kc + per * l;
     g.v_cache = m.vc + per * l;
-    gemm(c, g, st);
+    gemm(c, g, st, 0);
     AttnArgs a = {};
     a.T = T;
     a.n_heads = m.H;
@@ -464,7 +514,12 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     a.part_ml = m.part_ml;
     a.direct = p.prefill;
     a.err = c->err_word;
-    CK(attn_launch(a, m.mk[l], m.mv[l], st, pdl));
+    {
+      ProfScope ps(c, st, 5, 0.0, 0.0);
+      CK(attn_launch(a, m.mk[l], m.mv[l], st, pdl && !c->prof));
+      c->n_launch += a.direct ? 1 : 2;
+      ps.done();
+    }
     g = GemmArgs{};
     g.epi = EPI_RESID;
     g.W = m.wo[l];
@@ -475,8 +530,9 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.X_rows = m.Xrows;
     g.out_f32 = m.h;
     g.ldo = m.d;
-    gemm(c, g, st);
+    gemm(c, g, st, 1);
     CK(rmsnorm_launch(m.h, nullptr, nullptr, nullptr, m.mlp_norm[l], T, m.d, m.eps, m.x, m.d, st, pdl));
+    c->n_launch += 1;
     g = GemmArgs{};
     g.epi = EPI_SWIGLU;
     g.W = m.wgate_up[l];
@@ -487,7 +543,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.X_rows = m.Xrows;
     g.out_bf16 = m.act;
     g.ldo = m.ffn;
-    gemm(c, g, st);
+    gemm(c, g, st, 2);
     g = GemmArgs{};
     g.epi = EPI_RESID;
     g.W = m.wdown[l];
@@ -498,10 +554,11 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.X_rows = m.Xrows;
     g.out_f32 = m.h;
     g.ldo = m.d;
-    gemm(c, g, st);
+    gemm(c, g, st, 3);
   }
   const int n_out = (int)p.out_rows.size();
   CK(rmsnorm_rows_launch(m.h, m.rows_sel, n_out, m.final_norm, m.d, m.eps, m.x, m.d, st, pdl));
+  c->n_launch += 1;
   GemmArgs g = {};
   g.epi = EPI_F32;
   g.W = m.lm_head + (size_t)c->code_base * m.d;
@@ -512,7 +569,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
   g.X_rows = m.Xrows;
   g.out_f32 = m.logits + (size_t)p.logit_row_base * ITEM_ROWS;
   g.ldo = ITEM_ROWS;
-  gemm(c, g, st);
+  gemm(c, g, st, 4);
 }
 
 void add_qtiles(FwdPlan& p, int u, int t0, int n) {
@@ -537,6 +594,7 @@ void forward_nodes(atspeed_ctx* c, ModelRt& m, bool target, const std::vector<in
   CK(cudaMemcpyAsync(c->fwd_nodes, nodes.data(), T * 4, cudaMemcpyHostToDevice, st));
   FwdTokens f{m.tok, m.pos, m.kvrow, m.tuser, m.tvis, m.anc, m.ancn};
   CK(tree_gather_launch(t, c->fwd_nodes, T, c->u_P, c->code_base, target, row_base, f, st, c->pdl));
+  c->n_launch += 1;
   FwdPlan p;
   p.T = T;
   p.prefill = false;
@@ -713,6 +771,7 @@ void draft_step_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts*
   if (lvl > maxg) return;  // every tree is complete
   const TreeDev t = tree_dev(c);
   CK(draft_level_launch(t, lvl, c->step_N, mode == ATSPEED_RELAXED, o->philox_seed, st, c->pdl));
+  c->n_launch += 1;
   std::vector<int> nodes = level_nodes(c, lvl, true);
   // rows of this level's draft logits follow the rows already used in this step
   int base = c->B + (int)level_nodes(c, 0, false).size();
@@ -804,6 +863,7 @@ void verify_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts* o, 
   const TreeDev t = tree_dev(c);
   VerifyOut vo{c->o_acc, c->o_adv, c->o_n, c->o_nacc, c->o_path, c->o_score, c->o_parent, c->o_trie};
   CK(verify_launch(t, c->step_K, mode == ATSPEED_RELAXED, o->philox_seed, vo, st, c->pdl));
+  c->n_launch += 1;
   commit(c, st, true, T_user);
 }
 
@@ -1063,6 +1123,11 @@ void atspeed_destroy(atspeed_ctx* c) {
   if (!c) return;
   cudaSetDevice(c->device);
   cudaDeviceSynchronize();
+  for (auto& r : c->prof_recs) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (auto e : c->prof_pool) cudaEventDestroy(e);
   for (void* p : c->allocs) cudaFree(p);
   delete c;
 }
@@ -1176,6 +1241,47 @@ atspeed_status atspeed_begin_step(atspeed_ctx* c, atspeed_stream stream, const a
       throw Fail{ATSPEED_E_STATE};
     }
     ensure_step(c, opts, (cudaStream_t)stream);
+  });
+}
+
+atspeed_status atspeed_profile(atspeed_ctx* c, int enable) {
+  return guarded(c, [&] {
+    CK(cudaDeviceSynchronize());
+    for (auto& r : c->prof_recs) {
+      c->prof_pool.push_back(r.a);
+      c->prof_pool.push_back(r.b);
+    }
+    c->prof_recs.clear();
+    c->prof = enable != 0;
+  });
+}
+
+atspeed_status atspeed_profile_read(atspeed_ctx* c, int kind, int32_t* h_launches, double* h_ms, double* h_bytes,
+                                    double* h_flops) {
+  return guarded(c, [&] {
+    CK(cudaDeviceSynchronize());
+    if (kind < 0) {  // total kernel launches of this context since creation
+      if (h_launches) *h_launches = (int32_t)c->n_launch;
+      if (h_ms) *h_ms = 0;
+      if (h_bytes) *h_bytes = 0;
+      if (h_flops) *h_flops = 0;
+      return;
+    }
+    int n = 0;
+    double ms = 0, by = 0, fl = 0;
+    for (auto& r : c->prof_recs) {
+      if (r.kind != kind) continue;
+      float t = 0.f;
+      CK(cudaEventElapsedTime(&t, r.a, r.b));
+      ++n;
+      ms += t;
+      by += r.bytes;
+      fl += r.flops;
+    }
+    if (h_launches) *h_launches = n;
+    if (h_ms) *h_ms = ms;
+    if (h_bytes) *h_bytes = by;
+    if (h_flops) *h_flops = fl;
   });
 }
 

@@ -1,5 +1,5 @@
-// Shared-prefix tree attention: TMA-staged K/V pages, bf16 tensor cores (mma.sync m16n8k16) for
-// Q K^T and P V with an fp32 online softmax, prefix split across CTAs, then a combine kernel that
+// Shared-prefix tree attention: TMA-staged K/V pages, tensor cores (mma.sync m16n8k16: bf16 Q K^T;
+// P V with P split into two fp16 halves and V in fp16) with an fp32 online softmax, prefix split across CTAs, then a combine kernel that
 // merges the splits with each node's path keys (ancestors + self, at most 4).
 #include <cudaTypedefs.h>
 #include <math.h>
@@ -30,6 +30,21 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// p = hi + lo with hi = fp16(p) and lo = fp16(p - hi): 22 significant bits for the P V product.
+__device__ __forceinline__ void split_f16(float p0, float p1, uint32_t& hi, uint32_t& lo) {
+  const __half2 h = __floats2half2_rn(p0, p1);
+  const float2 hf = __half22float2(h);
+  const __half2 l = __floats2half2_rn(p0 - hf.x, p1 - hf.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -208,23 +223,18 @@ __global__ void __launch_bounds__(128)
       o[j][2] *= alpha_b;
       o[j][3] *= alpha_b;
     }
-    uint32_t pf[4][4];
+    uint32_t ph[4][4], pl[4][4];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const float p0 = exp2f(s[j][0] - ua), p1 = exp2f(s[j][1] - ua);
       const float p2 = exp2f(s[j][2] - ub), p3 = exp2f(s[j][3] - ub);
       l_a += p0 + p1;
       l_b += p2 + p3;
-      const int kk = j >> 1;
-      if ((j & 1) == 0) {
-        pf[kk][0] = pack_bf16(p0, p1);
-        pf[kk][1] = pack_bf16(p2, p3);
-      } else {
-        pf[kk][2] = pack_bf16(p0, p1);
-        pf[kk][3] = pack_bf16(p2, p3);
-      }
+      const int kk = j >> 1, r = (j & 1) * 2;
+      split_f16(p0, p1, ph[kk][r], pl[kk][r]);
+      split_f16(p2, p3, ph[kk][r + 1], pl[kk][r + 1]);
     }
-    // O += P V
+    // O += P V with P = hi + lo (fp16) and V fp16 (exactly the bf16-rounded values)
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk) {
 #pragma unroll
@@ -234,8 +244,10 @@ __global__ void __launch_bounds__(128)
         const int ch = dd * 2 + (lane >> 4);
         uint32_t b0, b1, b2, b3;
         ldsm_x4_t(vbase + kv_off<HD>(key, ch), b0, b1, b2, b3);
-        mma_bf16_16816(o[2 * dd], pf[kk], b0, b1);
-        mma_bf16_16816(o[2 * dd + 1], pf[kk], b2, b3);
+        mma_f16_16816(o[2 * dd], ph[kk], b0, b1);
+        mma_f16_16816(o[2 * dd + 1], ph[kk], b2, b3);
+        mma_f16_16816(o[2 * dd], pl[kk], b0, b1);
+        mma_f16_16816(o[2 * dd + 1], pl[kk], b2, b3);
       }
     }
     __syncthreads();  // buffer `buf` may be refilled next iteration
@@ -336,7 +348,7 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs a) {
     const float w = exp2f(sa[j] - Mu);
     L += w;
 #pragma unroll
-    for (int i = 0; i < PER; ++i) o[i] += w * __bfloat162float(a.v_cache[(size_t)row * d + h * HD + lane + 32 * i]);
+    for (int i = 0; i < PER; ++i) o[i] += w * __half2float(a.v_cache[(size_t)row * d + h * HD + lane + 32 * i]);
   }
   const float inv = L > 0.f ? 1.f / L : 0.f;
 #pragma unroll
@@ -389,7 +401,7 @@ cudaError_t launch_hd(const AttnArgs& a, const CUtensorMap& mk, const CUtensorMa
 
 }  // namespace
 
-bool attn_make_maps(const __nv_bfloat16* k_cache, const __nv_bfloat16* v_cache, int rows, int d_model, int head_dim,
+bool attn_make_maps(const __nv_bfloat16* k_cache, const __half* v_cache, int rows, int d_model, int head_dim,
                     CUtensorMap* mk, CUtensorMap* mv, char* eb, size_t el) {
   auto fn = encode_fn_att();
   if (!fn) {
@@ -403,8 +415,8 @@ bool attn_make_maps(const __nv_bfloat16* k_cache, const __nv_bfloat16* v_cache, 
   cuuint32_t es[2] = {1, 1};
   const CUtensorMapSwizzle sw = head_dim >= 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE;
   for (int i = 0; i < 2; ++i) {
-    CUresult r = fn(i == 0 ? mk : mv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-                    const_cast<__nv_bfloat16*>(i == 0 ? k_cache : v_cache), dims, strides, box, es,
+    CUresult r = fn(i == 0 ? mk : mv, i == 0 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2,
+                    i == 0 ? (void*)k_cache : (void*)v_cache, dims, strides, box, es,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) {

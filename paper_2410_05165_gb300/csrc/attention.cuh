@@ -7,6 +7,7 @@
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -20,7 +21,7 @@ struct AttnArgs {
   int T, n_heads, head_dim;        // d_model = n_heads * head_dim
   const __nv_bfloat16* q;          // [T][d] (RoPE applied)
   const __nv_bfloat16* k_cache;    // [rows][d] for this layer
-  const __nv_bfloat16* v_cache;
+  const __half* v_cache;           // fp16 holding bf16-rounded values (exact)
   int kv_rows;                     // rows of the cache arena
   // query tiles: consecutive tokens of one user
   int n_qtiles;
@@ -47,7 +48,7 @@ struct AttnArgs {
 };
 
 // Encodes the K/V tensor maps for one layer's cache arena (box = 64 rows x min(head_dim, 64)).
-bool attn_make_maps(const __nv_bfloat16* k_cache, const __nv_bfloat16* v_cache, int rows, int d_model,
+bool attn_make_maps(const __nv_bfloat16* k_cache, const __half* v_cache, int rows, int d_model,
                     int head_dim, CUtensorMap* mk, CUtensorMap* mv, char* eb, size_t el);
 
 cudaError_t attn_launch(const AttnArgs& a, const CUtensorMap& mk, const CUtensorMap& mv, cudaStream_t st, bool pdl);

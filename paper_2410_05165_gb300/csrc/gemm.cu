@@ -35,7 +35,7 @@ struct Cfg {
   static constexpr int B_BYTES = BN * 128;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGING_FLOATS = 32 * BM;
-  static constexpr int BAR_BYTES = 256;
+  static constexpr int BAR_BYTES = 256 + 1024;  // barriers, flags, split-part slot table
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_FLOATS * 4 + BAR_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
 };
@@ -90,7 +90,7 @@ __device__ __forceinline__ void epi_chunk(const KParams& p, const float* st, int
         const int region = row / d;
         const int f = row - region * d;
         if (region == 2) {
-          a.v_cache[(size_t)a.kv_row[tok] * d + f] = __float2bfloat16_rn(v);
+          a.v_cache[(size_t)a.kv_row[tok] * d + f] = __float2half_rn(bf16_round(v));
         } else {
           const int i = f % hd;
           const int ii = (i < half) ? i : i - half;
@@ -132,6 +132,7 @@ __global__ void __launch_bounds__(192, 1)
   int* flag = reinterpret_cast<int*>(tmem_slot + 1);
   int* failed = flag + 1;
   int* last_fill = failed + 1;  // [STAGES]: parity of the last fill issued per stage, -1 if none
+  int* part_slot = last_fill + 8;  // [<= 256] workspace slots of a split tile's parts
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x;
@@ -291,25 +292,25 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const int m_tile = tile / p.n_tiles, n_tile = tile % p.n_tiles;
       const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+      // 32-token chunks that hold at least one valid token (the rest are padding)
+      const int nch = min(BN / 32, (p.a.T - n_tile * BN + 31) / 32);
       if (k0 == 0 && k1 == kb) {
-        for (int ch = 0; ch < BN / 32; ++ch) {
+        for (int ch = 0; ch < nch; ++ch) {
           uint32_t r[32];
           tmem_ld_32x32b_x32(tb + ch * 32, r);
           tmem_ld_wait();
-          if (ch == BN / 32 - 1) {
-            tc_fence_before();
-            if (lane == 0) mbar_arrive(&tempty[acc]);
-          }
 #pragma unroll
           for (int j = 0; j < 32; ++j) staging[j * BM + m] = __uint_as_float(r[j]);
           named_bar_sync(1, 128);
           epi_chunk<BN, EPI>(p, staging, m_tile, n_tile, ch, ep_tid);
           named_bar_sync(1, 128);
         }
+        tc_fence_before();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
       } else {
         const long long slot = (long long)c * 2 + (si == 0 ? 0 : 1);
         float* wsl = p.ws + slot * WS_SLOT_FLOATS;
-        for (int ch = 0; ch < BN / 32; ++ch) {
+        for (int ch = 0; ch < nch; ++ch) {
           uint32_t r[32];
           tmem_ld_32x32b_x32(tb + ch * 32, r);
           tmem_ld_wait();
@@ -333,19 +334,27 @@ __global__ void __launch_bounds__(192, 1)
           }
           *flag = last;
         }
+        // workspace slot of every part, in k order
+        for (int pi = ep_tid; pi < parts; pi += 128) {
+          const int cc = c_first + pi;
+          part_slot[pi] = cc * 2 + (unit_start(cc, p.U, p.G) >= tu0 ? 0 : 1);
+        }
         named_bar_sync(1, 128);
         if (*flag) {
-          for (int ch = 0; ch < BN / 32; ++ch) {
-#pragma unroll 4
-            for (int j = 0; j < 32; ++j) {
-              float s = 0.0f;
-              for (int pi = 0; pi < parts; ++pi) {
-                const int cc = c_first + pi;
-                const long long sl = (long long)cc * 2 + (unit_start(cc, p.U, p.G) >= tu0 ? 0 : 1);
-                s += __ldcg(&p.ws[sl * WS_SLOT_FLOATS + (ch * 32 + j) * BM + m]);
-              }
-              staging[j * BM + m] = s;
+          for (int ch = 0; ch < nch; ++ch) {
+            float accv[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) accv[j] = 0.f;
+            for (int pi = 0; pi < parts; ++pi) {
+              const float* src = p.ws + (long long)part_slot[pi] * WS_SLOT_FLOATS + (ch * 32) * BM + m;
+              float v[32];
+#pragma unroll
+              for (int j = 0; j < 32; ++j) v[j] = __ldcg(src + j * BM);   // 32 independent loads in flight
+#pragma unroll
+              for (int j = 0; j < 32; ++j) accv[j] += v[j];
             }
+#pragma unroll
+            for (int j = 0; j < 32; ++j) staging[j * BM + m] = accv[j];
             named_bar_sync(1, 128);
             epi_chunk<BN, EPI>(p, staging, m_tile, n_tile, ch, ep_tid);
             named_bar_sync(1, 128);
@@ -451,7 +460,7 @@ int gemm_grid_size(int device) {
 
 cudaError_t gemm_launch(const GemmArgs& a, const GemmScratch& s, int grid, cudaStream_t stream, bool pdl,
                         char* eb, size_t el) {
-  if (a.K <= 0 || a.K % BK != 0 || a.M <= 0 || a.T <= 0) {
+  if (a.K <= 0 || a.K % BK != 0 || a.K / BK > 256 || a.M <= 0 || a.T <= 0) {
     snprintf(eb, el, "gemm: bad shape M=%d K=%d T=%d", a.M, a.K, a.T);
     return cudaErrorInvalidValue;
   }

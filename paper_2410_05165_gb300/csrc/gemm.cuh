@@ -2,6 +2,7 @@
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -33,7 +34,7 @@ struct GemmArgs {
   const float* rope_sin;
   __nv_bfloat16* q_out;     // [T][d_model]
   __nv_bfloat16* k_cache;   // [rows][d_model]
-  __nv_bfloat16* v_cache;
+  __half* v_cache;          // [rows][d_model]: v rounded to bf16, stored exactly as fp16
 };
 
 struct GemmScratch {

@@ -148,7 +148,7 @@ atspeed_status atspeed_op_attention(atspeed_stream stream, const void* d_q, cons
   const int d = n_heads * head_dim;
   CUtensorMap mk, mv;
   char eb[256];
-  if (!attn_make_maps(static_cast<const __nv_bfloat16*>(d_kcache), static_cast<const __nv_bfloat16*>(d_vcache),
+  if (!attn_make_maps(static_cast<const __nv_bfloat16*>(d_kcache), static_cast<const __half*>(d_vcache),
                       cache_rows, d, head_dim, &mk, &mv, eb, sizeof eb))
     return ATSPEED_E_CUDA;
   AttnArgs a = {};
@@ -157,7 +157,7 @@ atspeed_status atspeed_op_attention(atspeed_stream stream, const void* d_q, cons
   a.head_dim = head_dim;
   a.q = static_cast<const __nv_bfloat16*>(d_q);
   a.k_cache = static_cast<const __nv_bfloat16*>(d_kcache);
-  a.v_cache = static_cast<const __nv_bfloat16*>(d_vcache);
+  a.v_cache = static_cast<const __half*>(d_vcache);
   a.kv_rows = cache_rows;
   a.n_qtiles = nqt;
   const int off_qt0 = 0, off_qtn = nqt, off_qtu = 2 * nqt, off_tu = 3 * nqt, off_tv = off_tu + T, off_an = off_tv + T,

@@ -77,8 +77,10 @@ def test_swiglu_epilogue(ats, F, K, T):
     gu = X[:T].astype(np.float64) @ W.astype(np.float64).T
     ref = bf16(silu(gu[:, :F]) * gu[:, F:])
     err = np.abs(out - ref)
-    # one bf16 ulp (the fp32 pre-rounding value may sit on the other side of a rounding boundary)
-    assert np.all(err <= 2.0 ** -6 * np.abs(ref) + 1e-6), err.max()
+    # one bf16 ulp of the result, plus the fp32 accumulation error of g and u (absolute, ~1e-4 at
+    # K = 4096) carried through the product where g or u nearly cancels
+    g, u = gu[:, :F], gu[:, F:]
+    assert np.all(err <= 2.0 ** -6 * np.abs(ref) + 1e-4 * (np.abs(g) + np.abs(u) + 1.0)), err.max()
     assert np.mean(err > 0) < 0.01
 
 
@@ -87,7 +89,7 @@ def test_rmsnorm(ats, T, d):
     rng = np.random.default_rng(T + d)
     h = (rng.standard_normal((T, d)) * 3).astype(np.float32)
     g, gt = _bf16_tensor((d,), 5 + d, 0.1)
-    g = g + 1.0
+    g = bf16(g + 1.0).astype(np.float32)
     gt = torch.from_numpy(g).cuda().to(torch.bfloat16)
     x = ats.op_rmsnorm(torch.from_numpy(h).cuda(), gt, 1e-6).float().cpu().numpy()
     ref = bf16(rmsnorm(h.astype(np.float64), g.astype(np.float64), 1e-6))
@@ -114,7 +116,7 @@ def test_tree_attention(ats, H, hd, P, T):
     vis[: T // 3] = rng.integers(0, P + 1, size=T // 3)   # some causal-like partial visibility
     out = ats.op_attention(torch.from_numpy(q).cuda().to(torch.bfloat16),
                            torch.from_numpy(kc).cuda().to(torch.bfloat16),
-                           torch.from_numpy(vc).cuda().to(torch.bfloat16), H, hd, P, page_ids, vis, path_rows,
+                           torch.from_numpy(vc).cuda().to(torch.float16), H, hd, P, page_ids, vis, path_rows,
                            n_path).float().cpu().numpy()
     prefix_rows = np.array([64 * page_ids[p // 64] + p % 64 for p in range(P)], dtype=np.int64)
     for t in range(T):
@@ -125,4 +127,5 @@ def test_tree_attention(ats, H, hd, P, T):
         Kt = kc[keys].reshape(-1, H, hd).astype(np.float64)
         Vt = vc[keys].reshape(-1, H, hd).astype(np.float64)
         ref = _attend(q[t].reshape(1, H, hd).astype(np.float64), Kt, Vt, None)[0].reshape(-1)
-        assert np.abs(out[t] - ref).max() < 2e-2, (t, np.abs(out[t] - ref).max())
+        # fp32 softmax and P V with 22-bit P: only the final bf16 rounding of o remains
+        assert np.all(np.abs(out[t] - ref) <= 2.0 ** -7 * np.abs(ref) + 1e-5), (t, np.abs(out[t] - ref).max())
