@@ -214,6 +214,23 @@ size_t atspeed_op_workspace_bytes(void);
 atspeed_status atspeed_op_gemm(atspeed_stream stream, const void *d_W, const void *d_X, int M, int K, int T,
                                int x_rows, float *d_Y, int ldy, int accumulate, void *d_ws);
 
+/* Same result as atspeed_op_gemm, for callers that cannot allocate device memory: code that runs
+ * while a stream is being captured into a CUDA graph (an allocation there breaks or is not part of
+ * the capture), serving loops with a fixed, pre-reserved memory budget, and hosts whose device
+ * memory is owned by another allocator or pool that forbids direct cudaMalloc.  This entry point
+ * allocates nothing: its split-K scratch is a static device array inside this library, 8 MiB of
+ * partial sums (a 32-CTA grid, two 128 KiB slots per CTA) plus 16 KiB of tile counters and an error
+ * word, held by every GPU that loads the library until the process exits.  It therefore runs on at
+ * most 32 CTAs (slower than atspeed_op_gemm at large sizes) and accepts at most 4096 output tiles,
+ * ceil(M/128) * ceil(T/BN) with BN = 128 for T <= 128 and 256 above (ATSPEED_E_SHAPE otherwise),
+ * and K a multiple of 64 up to 16384.  Every call shares the one scratch array, which keeps the
+ * previous call's contents (the tile counters are cleared at the start of each call): calls that
+ * overlap on one GPU (issued on different streams, or from several host threads) race on it.  The
+ * first call on a device looks up the array's device address (no allocation); make that first call
+ * before any stream capture.  The paper has no counterpart: it is a deployment convenience. */
+atspeed_status atspeed_op_gemm_noalloc(atspeed_stream stream, const void *d_W, const void *d_X, int M, int K, int T,
+                                       int x_rows, float *d_Y, int ldy, int accumulate);
+
 /* out[t][j] = bf16(silu(G[t][j]) * U[t][j]) with G = X W[0:F]^T, U = X W[F:2F]^T (SwiGLU), W bf16
  * [2F][K]; out bf16 [T][ldo]. */
 atspeed_status atspeed_op_gemm_swiglu(atspeed_stream stream, const void *d_W, const void *d_X, int F, int K, int T,

@@ -26,7 +26,7 @@ EXPORTS = [
     "atspeed_draft_step", "atspeed_verify", "atspeed_draft_step_logits", "atspeed_verify_logits",
     "atspeed_beam_search", "atspeed_profile", "atspeed_profile_read", "atspeed_tree_shape", "atspeed_debug_tree",
     "atspeed_debug_node_logits", "atspeed_set_tree", "atspeed_op_workspace_bytes", "atspeed_op_gemm",
-    "atspeed_op_gemm_swiglu", "atspeed_op_rmsnorm", "atspeed_op_attention_scratch", "atspeed_op_attention",
+    "atspeed_op_gemm_noalloc", "atspeed_op_gemm_swiglu", "atspeed_op_rmsnorm", "atspeed_op_attention_scratch", "atspeed_op_attention",
 ]
 
 
@@ -95,6 +95,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "atspeed_set_tree": (c_int, [vp, vp, c_int, i32p, i32p, i32p, fp, fp]),
         "atspeed_op_workspace_bytes": (ctypes.c_size_t, []),
         "atspeed_op_gemm": (c_int, [vp, vp, vp, c_int, c_int, c_int, c_int, vp, c_int, c_int, vp]),
+        "atspeed_op_gemm_noalloc": (c_int, [vp, vp, vp, c_int, c_int, c_int, c_int, vp, c_int, c_int]),
         "atspeed_op_gemm_swiglu": (c_int, [vp, vp, vp, c_int, c_int, c_int, c_int, vp, c_int, vp]),
         "atspeed_op_rmsnorm": (c_int, [vp, vp, vp, c_int, c_int, ctypes.c_float, vp, c_int]),
         "atspeed_op_attention_scratch": (ctypes.c_size_t, [c_int, c_int, c_int, c_int]),
@@ -325,6 +326,17 @@ def op_gemm(W: torch.Tensor, X: torch.Tensor, T: int, Y: Optional[torch.Tensor] 
         Y = torch.zeros(T, M, dtype=torch.float32, device=W.device)
     _check(load().atspeed_op_gemm(_stream(stream), W.data_ptr(), X.data_ptr(), M, K, T, X.shape[0], Y.data_ptr(),
                                   Y.shape[1], 1 if accumulate else 0, op_workspace().data_ptr()))
+    return Y
+
+
+def op_gemm_noalloc(W: torch.Tensor, X: torch.Tensor, T: int, Y: Optional[torch.Tensor] = None, accumulate=False,
+                    stream=None) -> torch.Tensor:
+    """atspeed_op_gemm without a workspace argument (the library's fixed scratch array is used)."""
+    M, K = W.shape
+    if Y is None:
+        Y = torch.zeros(T, M, dtype=torch.float32, device=W.device)
+    _check(load().atspeed_op_gemm_noalloc(_stream(stream), W.data_ptr(), X.data_ptr(), M, K, T, X.shape[0],
+                                          Y.data_ptr(), Y.shape[1], 1 if accumulate else 0))
     return Y
 
 

@@ -5,6 +5,7 @@
 
 #include <algorithm>
 #include <cstring>
+#include <mutex>
 #include <vector>
 
 #include "atspeed.h"
@@ -40,6 +41,21 @@ atspeed_status run_gemm(cudaStream_t st, const GemmArgs& a, void* ws) {
   if (e == cudaErrorInvalidValue) return ATSPEED_E_SHAPE;
   return e == cudaSuccess ? ATSPEED_OK : ATSPEED_E_CUDA;
 }
+
+// ---------------------------------------------------------------------------------------------
+// Allocation-free GEMM: its split-K scratch lives in a fixed device array of this library.
+// ---------------------------------------------------------------------------------------------
+constexpr int kNoAllocGrid = 32;        // CTAs of the persistent grid (caps the workspace)
+constexpr int kNoAllocTiles = 4096;     // output tiles (128 weight rows x up to 256 tokens)
+constexpr size_t kNoAllocWsBytes = (size_t)2 * kNoAllocGrid * 256 * 128 * sizeof(float);  // 8 MiB
+constexpr size_t kNoAllocBytes = kNoAllocWsBytes + (size_t)kNoAllocTiles * sizeof(int) + 256;
+
+// One copy per GPU that loads the library, held until the process exits.  Host code must not use
+// this name as an address: the device address comes from cudaGetSymbolAddress (per device).
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[64] = {nullptr};
 
 }  // namespace
 
@@ -180,6 +196,51 @@ atspeed_status atspeed_op_attention(atspeed_stream stream, const void* d_q, cons
   a.direct = false;
   a.err = nullptr;
   const cudaError_t e = attn_launch(a, mk, mv, st, false);
+  return e == cudaSuccess ? ATSPEED_OK : ATSPEED_E_CUDA;
+}
+
+/* See include/atspeed.h.  The device address of the scratch array is looked up once per device, on
+ * that device's first call (so the first call on a device should come before any stream capture). */
+atspeed_status atspeed_op_gemm_noalloc(atspeed_stream stream, const void* d_W, const void* d_X, int M, int K, int T,
+                                       int x_rows, float* d_Y, int ldy, int accumulate) {
+  if (!d_W || !d_X || !d_Y || M <= 0 || K <= 0 || T <= 0 || ldy < M) return ATSPEED_E_ARG;
+  const int BN = T <= 128 ? 128 : 256;
+  const long long tiles = (long long)((M + 127) / 128) * ((T + BN - 1) / BN);
+  if (tiles > kNoAllocTiles || K % 64 != 0 || K / 64 > 256) return ATSPEED_E_SHAPE;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return ATSPEED_E_CUDA;
+  void* base = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+      void* ptr = nullptr;
+      if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return ATSPEED_E_CUDA;
+      g_noalloc_ptr[dev] = ptr;
+    }
+    base = g_noalloc_ptr[dev];
+  }
+  GemmScratch s;
+  s.ws = static_cast<float*>(base);
+  s.ws_bytes = kNoAllocWsBytes;
+  s.counters = reinterpret_cast<int*>(static_cast<char*>(base) + kNoAllocWsBytes);
+  s.max_tiles = kNoAllocTiles;
+  s.err = reinterpret_cast<unsigned int*>(static_cast<char*>(base) + kNoAllocWsBytes + (size_t)kNoAllocTiles * 4);
+  // the tile counters must start at zero (a call that failed part-way could have left some set)
+  if (cudaMemsetAsync(s.counters, 0, (size_t)kNoAllocTiles * sizeof(int), (cudaStream_t)stream) != cudaSuccess)
+    return ATSPEED_E_CUDA;
+  GemmArgs a = {};
+  a.epi = accumulate ? EPI_RESID : EPI_F32;
+  a.W = static_cast<const __nv_bfloat16*>(d_W);
+  a.X = static_cast<const __nv_bfloat16*>(d_X);
+  a.M = M;
+  a.K = K;
+  a.T = T;
+  a.X_rows = x_rows;
+  a.out_f32 = d_Y;
+  a.ldo = ldy;
+  char eb[256];
+  const cudaError_t e = gemm_launch(a, s, kNoAllocGrid, (cudaStream_t)stream, false, eb, sizeof eb);
+  if (e == cudaErrorInvalidValue) return ATSPEED_E_SHAPE;
   return e == cudaSuccess ? ATSPEED_OK : ATSPEED_E_CUDA;
 }
 
