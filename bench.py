@@ -42,6 +42,10 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="7b")
     ap.add_argument("--mode", choices=["strict", "relaxed"], default="strict")
+    ap.add_argument("--verify-only", type=int, default=0, metavar="R",
+                    help="profiling aid: R verification calls of the workload, each in an NVTX range 'verify'")
+    ap.add_argument("--kernel-probe", action="store_true",
+                    help="profiling aid: the four layer GEMMs of the 7B shape at T=120 over 8 layers of weights")
     return ap.parse_args()
 
 
@@ -315,9 +319,81 @@ def run_ours(args, w):
         dist.destroy_process_group()
 
 
+def kernel_probe():
+    """The weight-streaming GEMM alone at the verification call's shapes (T = 120 tree tokens),
+    over 8 layers of distinct weights (3.2 GB, larger than L2), timed with CUDA events."""
+    import torch
+    import paper_2410_05165_gb300 as ats
+    ats.load()
+    d, f, T, nl = 4096, 11008, 120, 8
+    shapes = {"qkv": (3 * d, d), "o": (d, d), "gate_up": (2 * f, d), "down": (d, f)}
+    g = torch.Generator(device="cuda").manual_seed(0)
+    Ws = {k: [(torch.randn(m, kk, device="cuda", generator=g) * 0.02).to(torch.bfloat16) for _ in range(nl)]
+          for k, (m, kk) in shapes.items()}
+    X = {kk: torch.randn(256, kk, device="cuda", generator=g).to(torch.bfloat16) for kk in (d, f)}
+    out = {}
+    for k, (m, kk) in shapes.items():
+        Y = torch.zeros(T, m, device="cuda")
+        ts = []
+        for rep in range(3):
+            for l in range(nl):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                ats.op_gemm(Ws[k][l], X[kk], T, Y=Y)
+                e1.record()
+                torch.cuda.synchronize()
+                if rep:
+                    ts.append(e0.elapsed_time(e1))
+        t = statistics.median(ts)
+        out[k] = {"M": m, "K": kk, "us": t * 1e3, "weight_GBps": m * kk * 2 / (t / 1e3) / 1e9}
+    print(json.dumps({"kernel_probe": out}), flush=True)
+
+
+def verify_only(w, mode, reps):
+    import torch
+    import paper_2410_05165_gb300 as ats
+    ats.load()
+    tw = {n: torch.from_numpy(a).to(device="cuda", dtype=torch.bfloat16)
+          for n, a in synth.iter_model_tensors(w.target, w.seed, "target")}
+    dw = {n: torch.from_numpy(a).to(device="cuda", dtype=torch.bfloat16)
+          for n, a in synth.iter_model_tensors(w.draft, w.seed, "draft")}
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    prompts = synth.make_prompts(w.n_users, w.prompt_len, w.target.vocab, w.seed)
+    P = [len(p) for p in prompts]
+    ctx = ats.Context(w.target, tw, w.draft, dw, items, w.code_base, max_users=len(prompts), max_prompt=max(P),
+                      max_K=w.K, max_N=w.N, max_gamma=w.gamma)
+    toks = torch.from_numpy(np.concatenate(prompts).astype(np.int32)).cuda()
+    off = np.concatenate([[0], np.cumsum(P)]).astype(np.int32)
+    o = ats.opts(w.K, w.N, w.gamma, w.philox_seed)
+    vm = ats.STRICT if mode == "strict" else ats.RELAXED
+    ms = []
+    for r in range(reps):
+        ctx.prefill(toks, off)
+        ctx.begin_step(o)
+        for _ in range(w.gamma):
+            ctx.draft_step(o, vm)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.nvtx.range_push("verify")
+        e0.record()
+        ctx.verify(o, vm)
+        e1.record()
+        torch.cuda.nvtx.range_pop()
+        torch.cuda.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    print(json.dumps({"verify_ms": ms}), flush=True)
+    ctx.close()
+
+
 def main():
     args = parse()
     w = synth.workload(args.workload)
+    if args.kernel_probe:
+        kernel_probe()
+        return
+    if args.verify_only:
+        verify_only(w, args.mode, args.verify_only)
+        return
     if args.impl == "reference":
         run_reference(args, w)
     else:
