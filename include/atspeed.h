@@ -169,12 +169,20 @@ atspeed_status atspeed_beam_search(atspeed_ctx *ctx, atspeed_stream stream, int 
  * CUDA events on its stream (and programmatic dependent launch is off, so launches do not
  * overlap).  atspeed_profile(ctx, 1) clears previous records.  profile_read sums, over the
  * launches of one kind (0 QKV GEMM, 1 O GEMM, 2 gate/up GEMM, 3 down GEMM, 4 LM-head GEMM,
- * 5 attention), the launch count, the device time (ms), and the algorithmic bytes and FLOPs (weights
+ * 5 attention, 6 whole persistent forward kernel), the launch count, the device time (ms), and the algorithmic bytes and FLOPs (weights
  * read once, activations in, outputs out).  kind < 0 returns in *h_launches the number of kernels
  * the context has launched since creation (every kind, profiling on or off).  Synchronises. */
 atspeed_status atspeed_profile(atspeed_ctx *ctx, int enable);
 atspeed_status atspeed_profile_read(atspeed_ctx *ctx, int kind, int32_t *h_launches, double *h_ms, double *h_bytes,
                                     double *h_flops);
+
+/* Copies the first `bytes` of one internal buffer of the target (which = 0) or draft (1) decoder
+ * to the host: id 0 residual stream h (fp32 [T][d]), 1 normalised rows x (bf16), 2 q (bf16),
+ * 3 attention output (bf16), 4 SwiGLU output (bf16 [T][d_ffn]), 5 K cache (bf16, all layers),
+ * 6 V cache (fp16), 7 item-code logits (fp32 [rows][1024]), 8 the persistent forward's barrier
+ * counter (u32), 9 its per-phase timestamps ([phases][CTAs] u64 ns, recorded only when the
+ * environment variable ATSPEED_FWD_TRACE=1 was set at create time).  Synchronises the device. */
+atspeed_status atspeed_debug_buffer(atspeed_ctx *ctx, int which, int id, void *h_out, size_t bytes);
 
 /* Shape of the current speculative step: h_depth[n_users], h_levels[n_users] (drafted levels),
  * and the node-table geometry (*h_slots_in slots on level 0, *h_slots_lvl per drafted level). */

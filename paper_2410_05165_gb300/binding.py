@@ -25,7 +25,7 @@ EXPORTS = [
     "atspeed_create", "atspeed_destroy", "atspeed_last_error", "atspeed_prefill", "atspeed_begin_step",
     "atspeed_draft_step", "atspeed_verify", "atspeed_draft_step_logits", "atspeed_verify_logits",
     "atspeed_beam_search", "atspeed_profile", "atspeed_profile_read", "atspeed_tree_shape", "atspeed_debug_tree",
-    "atspeed_debug_node_logits", "atspeed_set_tree", "atspeed_op_workspace_bytes", "atspeed_op_gemm",
+    "atspeed_debug_node_logits", "atspeed_debug_buffer", "atspeed_set_tree", "atspeed_op_workspace_bytes", "atspeed_op_gemm",
     "atspeed_op_gemm_noalloc", "atspeed_op_gemm_swiglu", "atspeed_op_rmsnorm", "atspeed_op_attention_scratch", "atspeed_op_attention",
 ]
 
@@ -92,6 +92,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "atspeed_tree_shape": (c_int, [vp, i32p, i32p, i32p, i32p]),
         "atspeed_debug_tree": (c_int, [vp, i32p, fp, fp, i32p]),
         "atspeed_debug_node_logits": (c_int, [vp, c_int, c_int, c_int, fp]),
+        "atspeed_debug_buffer": (c_int, [vp, c_int, c_int, vp, ctypes.c_size_t]),
         "atspeed_set_tree": (c_int, [vp, vp, c_int, i32p, i32p, i32p, fp, fp]),
         "atspeed_op_workspace_bytes": (ctypes.c_size_t, []),
         "atspeed_op_gemm": (c_int, [vp, vp, vp, c_int, c_int, c_int, c_int, vp, c_int, c_int, vp]),
@@ -283,6 +284,11 @@ class Context:
                                             cnt.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))), self.ptr)
         return {"path": path, "sq": sq, "sp": sp, "count": cnt, "slots_in": si, "slots_lvl": sl, "depth": depth,
                 "levels": levels}
+
+    def debug_buffer(self, which: int, buf: int, dtype, count: int) -> np.ndarray:
+        out = np.zeros(count, dtype=dtype)
+        _check(self._lib.atspeed_debug_buffer(self.ptr, which, buf, out.ctypes.data, out.nbytes), self.ptr)
+        return out
 
     def node_logits(self, which: int, user: int, slot: int) -> np.ndarray:
         out = np.zeros(1024, np.float32)

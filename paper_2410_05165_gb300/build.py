@@ -18,7 +18,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libatspeed.so")
 
-SOURCES = ["api.cu", "ops.cu", "gemm.cu", "attention.cu", "norm.cu", "select.cu", "tree_ops.cu"]
+SOURCES = ["api.cu", "ops.cu", "gemm.cu", "attention.cu", "norm.cu", "select.cu", "tree_ops.cu", "fwd.cu"]
+EXTRA = {}
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC,
          "--expt-relaxed-constexpr", "-diag-suppress", "177"]
@@ -48,7 +49,7 @@ def build(verbose: bool = False, force: bool = False) -> str:
         src = os.path.join(CSRC, s)
         obj = os.path.join(BUILD, s.replace(".cu", ".o"))
         if force or _stale(obj, src):
-            jobs.append([cc, *ARCH, *FLAGS, "-c", src, "-o", obj])
+            jobs.append([cc, *ARCH, *FLAGS, *EXTRA.get(s, []), "-c", src, "-o", obj])
 
     def run(cmd):
         r = subprocess.run(cmd, capture_output=True, text=True)

@@ -9,6 +9,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -16,6 +17,7 @@
 #include "atspeed.h"
 #include "common.cuh"
 #include "attention.cuh"
+#include "fwd.cuh"
 #include "gemm.cuh"
 #include "kernels.cuh"
 #include "tree.cuh"
@@ -58,6 +60,12 @@ struct ModelRt {
   int *qt_t0 = nullptr, *qt_n = nullptr, *qt_user = nullptr, *rows_sel = nullptr, *user_splits = nullptr;
   float *part_o = nullptr, *part_ml = nullptr;
   int max_splits = 1;
+  // persistent forward kernel
+  CUtensorMap* maps = nullptr;           // device table, layout in fwd.cuh
+  const bf16** d_attn_norm = nullptr;    // device arrays of layer pointers
+  const bf16** d_mlp_norm = nullptr;
+  int* att_counters = nullptr;
+  int max_qt = 0;
 };
 
 struct UserState {
@@ -126,6 +134,11 @@ struct atspeed_ctx {
   std::vector<ProfRec> prof_recs;
   std::vector<cudaEvent_t> prof_pool;
   long long n_launch = 0;  // kernels launched by this context (all kinds)
+  bool per_op = true;      // one kernel per op (else the persistent single-launch forward)
+  int fwd_grid = 0;
+  unsigned int* fwd_bar = nullptr;
+  unsigned long long* fwd_trace = nullptr;  // per-phase timestamps of the last forward (tracing on)
+  size_t fwd_trace_n = 0;
 };
 
 namespace {
@@ -197,8 +210,8 @@ void init_model(atspeed_ctx* c, ModelRt& m, const atspeed_model_desc* md, const 
     set_err(c, "%s: head_dim %d not in {32, 64, 128}", name, hd);
     throw Fail{ATSPEED_E_SHAPE};
   }
-  if (md->d_model % 64 || md->d_ffn % 64) {
-    set_err(c, "%s: d_model and d_ffn must be multiples of 64", name);
+  if (md->d_model % 64 || md->d_ffn % 64 || md->d_model > 8192) {
+    set_err(c, "%s: d_model and d_ffn must be multiples of 64, d_model at most 8192", name);
     throw Fail{ATSPEED_E_SHAPE};
   }
   if (!md->embed || !md->final_norm || !md->lm_head || !md->attn_norm || !md->wqkv || !md->wo || !md->mlp_norm ||
@@ -242,12 +255,14 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.vc = dalloc<__half>(c, per * m.layers);
   m.mk.resize(m.layers);
   m.mv.resize(m.layers);
+  {
   char eb[256];
   for (int l = 0; l < m.layers; ++l)
     if (!attn_make_maps(m.kc + per * l, m.vc + per * l, m.rows, m.d, m.hd, &m.mk[l], &m.mv[l], eb, sizeof eb)) {
       set_err(c, "%s", eb);
       throw Fail{ATSPEED_E_CUDA};
     }
+  }
   // rotary tables, computed in double precision
   m.max_pos = L.max_prompt + TREE_L + 1;
   const int half = m.hd / 2;
@@ -280,6 +295,7 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.anc = dalloc<int>(c, (size_t)m.Tcap * 4);
   m.ancn = dalloc<int>(c, m.Tcap);
   const int max_qt = m.Tcap / ATT_QTILE + L.max_users + 1;
+  char eb[256];
   m.qt_t0 = dalloc<int>(c, max_qt);
   m.qt_n = dalloc<int>(c, max_qt);
   m.qt_user = dalloc<int>(c, max_qt);
@@ -287,9 +303,44 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.user_splits = dalloc<int>(c, L.max_users);
   const int pages = c->prefix_pages_per_user;
   m.max_splits = std::max(1, (pages + kChunksPerSplit - 1) / kChunksPerSplit);
-  const int Ttree = L.max_users * stride;
+  const int Ttree = std::max(L.max_users * stride, m.Tcap);
   m.part_o = dalloc<float>(c, (size_t)m.max_splits * Ttree * m.d, false);
   m.part_ml = dalloc<float>(c, (size_t)m.max_splits * Ttree * m.H * 2, false);
+  m.max_qt = max_qt;
+  m.att_counters = dalloc<int>(c, (size_t)max_qt * m.H);
+  // tensor maps of the persistent forward
+  const int nmaps = fwd_map_count(m.layers);
+  std::vector<CUtensorMap> hm(nmaps);
+  for (int l = 0; l < m.layers; ++l) {
+    const bool ok = gemm_make_map(&hm[l * 4 + 0], m.wqkv[l], m.d, 3 * m.d, 64, eb, sizeof eb) &&
+                    gemm_make_map(&hm[l * 4 + 1], m.wo[l], m.d, m.d, 64, eb, sizeof eb) &&
+                    gemm_make_map(&hm[l * 4 + 2], m.wgate_up[l], m.d, 2 * m.ffn, 64, eb, sizeof eb) &&
+                    gemm_make_map(&hm[l * 4 + 3], m.wdown[l], m.ffn, m.d, 64, eb, sizeof eb);
+    if (!ok) {
+      set_err(c, "%s", eb);
+      throw Fail{ATSPEED_E_CUDA};
+    }
+    hm[4 * m.layers + 2 * l] = m.mk[l];
+    hm[4 * m.layers + 2 * l + 1] = m.mv[l];
+  }
+  const int L6 = 6 * m.layers;
+  bool ok = gemm_make_map(&hm[L6], m.lm_head + (size_t)c->code_base * m.d, m.d, ITEM_ROWS, 64, eb, sizeof eb);
+  for (int v = 0; v < 2 && ok; ++v) {
+    const int bn = v == 0 ? 128 : 256;
+    ok = gemm_make_map(&hm[L6 + 1 + 3 * v], m.x, m.d, m.Xrows, bn, eb, sizeof eb) &&
+         gemm_make_map(&hm[L6 + 2 + 3 * v], m.att, m.d, m.Xrows, bn, eb, sizeof eb) &&
+         gemm_make_map(&hm[L6 + 3 + 3 * v], m.act, m.ffn, m.Xrows, bn, eb, sizeof eb);
+  }
+  if (!ok) {
+    set_err(c, "%s", eb);
+    throw Fail{ATSPEED_E_CUDA};
+  }
+  m.maps = dalloc<CUtensorMap>(c, nmaps, false);
+  CK(cudaMemcpy(m.maps, hm.data(), nmaps * sizeof(CUtensorMap), cudaMemcpyHostToDevice));
+  m.d_attn_norm = dalloc<const bf16*>(c, m.layers, false);
+  m.d_mlp_norm = dalloc<const bf16*>(c, m.layers, false);
+  CK(cudaMemcpy(m.d_attn_norm, m.attn_norm.data(), m.layers * sizeof(void*), cudaMemcpyHostToDevice));
+  CK(cudaMemcpy(m.d_mlp_norm, m.mlp_norm.data(), m.layers * sizeof(void*), cudaMemcpyHostToDevice));
 }
 
 void build_trie(atspeed_ctx* c, const atspeed_items_desc* it) {
@@ -466,6 +517,81 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
   for (int s : p.splits) max_split = std::max(max_split, s);
   const size_t per = (size_t)m.rows * m.d;
   const bool pdl = c->pdl;
+  if (!c->per_op) {
+    // the whole forward in one persistent cooperative launch
+    if (nqt > m.max_qt) {
+      set_err(c, "forward needs %d query tiles (capacity %d)", nqt, m.max_qt);
+      throw Fail{ATSPEED_E_SHAPE};
+    }
+    FwdParams f = {};
+    f.T = T;
+    f.n_out = (int)p.out_rows.size();
+    f.d = m.d;
+    f.H = m.H;
+    f.hd = m.hd;
+    f.ffn = m.ffn;
+    f.L = m.layers;
+    f.eps = m.eps;
+    f.G = c->fwd_grid;
+    f.maps = m.maps;
+    f.attn_norm = m.d_attn_norm;
+    f.mlp_norm = m.d_mlp_norm;
+    f.final_norm = m.final_norm;
+    f.embed = m.embed;
+    f.h = m.h;
+    f.x = m.x;
+    f.q = m.q;
+    f.att = m.att;
+    f.act = m.act;
+    f.logits = m.logits + (size_t)p.logit_row_base * ITEM_ROWS;
+    f.kc = m.kc;
+    f.vc = m.vc;
+    f.layer_elems = per;
+    f.tok = p.d_tokens;
+    f.pos = m.pos;
+    f.kv_row = m.kvrow;
+    f.out_rows = m.rows_sel;
+    f.rope_cos = m.rope_cos;
+    f.rope_sin = m.rope_sin;
+    AttnArgs& a = f.att_args;
+    a.T = T;
+    a.n_heads = m.H;
+    a.head_dim = m.hd;
+    a.q = m.q;
+    a.kv_rows = m.rows;
+    a.n_qtiles = nqt;
+    a.qt_t0 = m.qt_t0;
+    a.qt_n = m.qt_n;
+    a.qt_user = m.qt_user;
+    a.tok_user = m.tuser;
+    a.tok_vis = m.tvis;
+    a.anc_row = p.prefill ? nullptr : m.anc;
+    a.anc_n = p.prefill ? nullptr : m.ancn;
+    a.page_table = c->page_table;
+    a.max_pages = c->prefix_pages_per_user;
+    a.user_splits = m.user_splits;
+    a.chunks_per_split = p.prefill ? 0 : kChunksPerSplit;
+    a.max_splits = max_split;
+    a.out = m.att;
+    a.part_o = m.part_o;
+    a.part_ml = m.part_ml;
+    a.direct = p.prefill;
+    a.err = c->err_word;
+    f.att_items = nqt * m.H * max_split;
+    f.att_counters = m.att_counters;
+    f.ws = c->gs.ws;
+    f.counters = c->gs.counters;
+    f.bar = c->fwd_bar;
+    f.err = c->err_word;
+    f.trace = c->fwd_trace;
+    CK(cudaMemsetAsync(c->fwd_bar, 0, sizeof(unsigned int), st));
+    const double wbytes = 2.0 * m.layers * (4.0 * m.d * m.d + 3.0 * m.d * m.ffn) + 2.0 * ITEM_ROWS * m.d;
+    ProfScope ps(c, st, 6, wbytes, 2.0 * T * (wbytes / 2.0));
+    CK(fwd_launch(f, st));
+    ps.done();
+    c->n_launch += 1;
+    return;
+  }
   for (int l = 0; l < m.layers; ++l) {
     CK(rmsnorm_launch(m.h, l == 0 ? p.d_tokens : nullptr, m.embed, m.h, m.attn_norm[l], T, m.d, m.eps, m.x, m.d, st,
                       pdl));
@@ -1071,6 +1197,21 @@ atspeed_status atspeed_create(const atspeed_model_desc* target, const atspeed_mo
     alloc_model(c, c->tgt);
     alloc_model(c, c->drf);
     c->gemm_grid = gemm_grid_size(c->device);
+    c->fwd_grid = c->gemm_grid;  // one persistent CTA per SM
+    {
+      // ATSPEED_FORWARD=persistent selects the single-launch forward; the default is one kernel per op
+      const char* fm = getenv("ATSPEED_FORWARD");
+      c->per_op = !(fm && strcmp(fm, "persistent") == 0);
+    }
+    c->fwd_bar = dalloc<unsigned int>(c, 1);
+    {
+      const char* tr = getenv("ATSPEED_FWD_TRACE");
+      if (tr && tr[0] == '1') {
+        const int Lmax = std::max(c->tgt.layers, c->drf.present ? c->drf.layers : 0);
+        c->fwd_trace_n = (size_t)4 * (7 * Lmax + 2) * c->fwd_grid;
+        c->fwd_trace = dalloc<unsigned long long>(c, c->fwd_trace_n);
+      }
+    }
     c->gs.ws_bytes = gemm_ws_bytes(c->gemm_grid);
     c->gs.ws = dalloc<float>(c, c->gs.ws_bytes / 4, false);
     c->gs.max_tiles = gemm_max_tiles();
@@ -1282,6 +1423,33 @@ atspeed_status atspeed_profile_read(atspeed_ctx* c, int kind, int32_t* h_launche
     if (h_ms) *h_ms = ms;
     if (h_bytes) *h_bytes = by;
     if (h_flops) *h_flops = fl;
+  });
+}
+
+atspeed_status atspeed_debug_buffer(atspeed_ctx* c, int which, int id, void* h_out, size_t bytes) {
+  return guarded(c, [&] {
+    const ModelRt& m = which == 0 ? c->tgt : c->drf;
+    const void* src = nullptr;
+    size_t cap = 0;
+    switch (id) {
+      case 0: src = m.h; cap = (size_t)m.Tcap * m.d * 4; break;
+      case 1: src = m.x; cap = (size_t)m.Xrows * m.d * 2; break;
+      case 2: src = m.q; cap = (size_t)m.Tcap * m.d * 2; break;
+      case 3: src = m.att; cap = (size_t)m.Xrows * m.d * 2; break;
+      case 4: src = m.act; cap = (size_t)m.Xrows * m.ffn * 2; break;
+      case 5: src = m.kc; cap = (size_t)m.rows * m.d * 2 * m.layers; break;
+      case 6: src = m.vc; cap = (size_t)m.rows * m.d * 2 * m.layers; break;
+      case 7: src = m.logits; cap = (size_t)m.logit_rows * ITEM_ROWS * 4; break;
+      case 8: src = c->fwd_bar; cap = 4; break;
+      case 9: src = c->fwd_trace; cap = c->fwd_trace_n * 8; break;
+      default: break;
+    }
+    if (!m.present || !src || !h_out || bytes > cap) {
+      set_err(c, "debug_buffer: bad arguments");
+      throw Fail{ATSPEED_E_ARG};
+    }
+    CK(cudaDeviceSynchronize());
+    CK(cudaMemcpy(h_out, src, bytes, cudaMemcpyDeviceToHost));
   });
 }
 

@@ -6,353 +6,42 @@
 #include <stdio.h>
 
 #include "attention.cuh"
+#include "attn_core.cuh"
 #include "common.cuh"
 
 namespace atspeed {
 
 namespace {
 
-constexpr float kLog2e = 1.4426950408889634f;
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-// p = hi + lo with hi = fp16(p) and lo = fp16(p - hi): 22 significant bits for the P V product.
-__device__ __forceinline__ void split_f16(float p0, float p1, uint32_t& hi, uint32_t& lo) {
-  const __half2 h = __floats2half2_rn(p0, p1);
-  const float2 hf = __half22float2(h);
-  const __half2 l = __floats2half2_rn(p0 - hf.x, p1 - hf.y);
-  hi = *reinterpret_cast<const uint32_t*>(&h);
-  lo = *reinterpret_cast<const uint32_t*>(&l);
-}
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
-}
-
-// Byte offset of (row, 16-byte chunk) inside a K or V page tile as written by TMA.
-// HD >= 64: boxes of 64 columns (128 B rows), 128-byte swizzle: chunk ^= row & 7.
-// HD == 32: one box of 64-byte rows, no swizzle.
-template <int HD>
-__device__ __forceinline__ uint32_t kv_off(int row, int chunk16) {
-  if constexpr (HD >= 64) {
-    const int box = chunk16 >> 3, c = chunk16 & 7;
-    return (uint32_t)(box * (ATT_PAGE * 128) + row * 128 + ((c ^ (row & 7)) << 4));
-  } else {
-    return (uint32_t)(row * (HD * 2) + (chunk16 << 4));
-  }
-}
-
-template <int HD>
-struct AttCfg {
-  static constexpr int QSTRIDE = HD + 8;                    // bf16 elements per Q row in smem
-  static constexpr int Q_BYTES = ATT_QTILE * QSTRIDE * 2;
-  static constexpr int KV_BYTES = ATT_PAGE * HD * 2;         // one K (or V) page tile
-  static constexpr int BUF_BYTES = 2 * KV_BYTES;             // K + V
-  static constexpr int SMEM = 1024 + 2 * BUF_BYTES + Q_BYTES + 64;
-};
-
 template <int HD>
 __global__ void __launch_bounds__(128)
     attn_prefix_kernel(const __grid_constant__ CUtensorMap mk, const __grid_constant__ CUtensorMap mv,
                        const AttnArgs a) {
   using C = AttCfg<HD>;
-  constexpr int NDT = HD / 8;    // dim n-tiles of O
-  constexpr int NKS = HD / 16;   // k-steps of Q K^T
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* kvbuf = smem;                                             // [2][K | V]
-  __nv_bfloat16* qs = reinterpret_cast<__nv_bfloat16*>(smem + 2 * C::BUF_BYTES);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 2 * C::BUF_BYTES + C::Q_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::SMEM_BODY);
   int* s_info = reinterpret_cast<int*>(bars + 2);
-
-  const int tile = blockIdx.x, h = blockIdx.y, split = blockIdx.z;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int d = a.n_heads * HD;
-
   pdl_launch_dependents();
   pdl_wait();
-  const int u = a.qt_user[tile];
-  const int t0 = a.qt_t0[tile];
-  const int nq = a.qt_n[tile];
-  const int S_u = a.user_splits[u];
-  if (split >= S_u) return;
-
-  if (tid == 0) {
-    int mv_ = 0;
-    for (int i = 0; i < nq; ++i) mv_ = max(mv_, a.tok_vis[t0 + i]);
-    const int nch = (mv_ + ATT_PAGE - 1) / ATT_PAGE;
-    int c0 = 0, c1 = nch;
-    if (a.chunks_per_split > 0) {
-      c0 = min(nch, split * a.chunks_per_split);
-      c1 = min(nch, c0 + a.chunks_per_split);
-    }
-    s_info[0] = c0;
-    s_info[1] = c1;
+  if (threadIdx.x == 0) {
     mbar_init(&bars[0], 1);
     mbar_init(&bars[1], 1);
     fence_mbar_init();
-  }
-  // Q tile -> shared memory (rows >= nq are zero)
-  for (int i = tid; i < ATT_QTILE * (HD / 8); i += 128) {
-    const int r = i / (HD / 8), c = i % (HD / 8);
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (r < nq) v = *reinterpret_cast<const uint4*>(a.q + (size_t)(t0 + r) * d + h * HD + c * 8);
-    *reinterpret_cast<uint4*>(qs + r * C::QSTRIDE + c * 8) = v;
-  }
-  __syncthreads();
-  const int c0 = s_info[0], c1 = s_info[1];
-  const int* ptab = a.page_table + (size_t)u * a.max_pages;
-  constexpr int NBOX = HD >= 64 ? HD / 64 : 1;
-  constexpr int BOXW = HD >= 64 ? 64 : HD;
-
-  auto issue = [&](int chunk, int buf) {
-    const int row0 = ptab[chunk] * ATT_PAGE;
-    uint8_t* kb = kvbuf + buf * C::BUF_BYTES;
-    mbar_arrive_expect_tx(&bars[buf], C::BUF_BYTES);
-    const uint64_t pol = policy_evict_last();
-    for (int b = 0; b < NBOX; ++b) {
-      tma_load_2d(kb + b * (ATT_PAGE * BOXW * 2), &mk, &bars[buf], h * HD + b * BOXW, row0, pol);
-      tma_load_2d(kb + C::KV_BYTES + b * (ATT_PAGE * BOXW * 2), &mv, &bars[buf], h * HD + b * BOXW, row0, pol);
-    }
-  };
-  if (tid == 0 && c0 < c1) {
     tma_prefetch_desc(&mk);
     tma_prefetch_desc(&mv);
-    issue(c0, 0);
   }
-
-  // Q fragments (A operand) for this warp's 16 rows
-  uint32_t qf[NKS][4];
-  {
-    const uint32_t qbase = smem_u32(qs);
-    const int r = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-    const int cofs = (lane >> 4) * 8;
-#pragma unroll
-    for (int kk = 0; kk < NKS; ++kk)
-      ldsm_x4(qbase + (uint32_t)((r * C::QSTRIDE + kk * 16 + cofs) * 2), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
-  }
-  const int g = lane >> 2, tq = lane & 3;
-  const int row_a = warp * 16 + g, row_b = row_a + 8;
-  const int vis_a = row_a < nq ? a.tok_vis[t0 + row_a] : 0;
-  const int vis_b = row_b < nq ? a.tok_vis[t0 + row_b] : 0;
-  const float scale = kLog2e / sqrtf((float)HD);
-
-  float o[NDT][4];
-#pragma unroll
-  for (int j = 0; j < NDT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
-  float m_a = -INFINITY, m_b = -INFINITY, l_a = 0.f, l_b = 0.f;
-  bool ok = true;
-
-  for (int chunk = c0; chunk < c1; ++chunk) {
-    const int buf = (chunk - c0) & 1;
-    if (tid == 0 && chunk + 1 < c1) issue(chunk + 1, buf ^ 1);
-    const bool got = mbar_wait(&bars[buf], (uint32_t)(((chunk - c0) >> 1) & 1), a.err);
-    __syncwarp();
-    if (!got) {
-      ok = false;
-      break;
-    }
-    const uint32_t kbase = smem_u32(kvbuf + buf * C::BUF_BYTES);
-    const uint32_t vbase = kbase + C::KV_BYTES;
-    float s[8][4];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
-#pragma unroll
-    for (int jj = 0; jj < 4; ++jj) {
-#pragma unroll
-      for (int kk = 0; kk < NKS; ++kk) {
-        // matrices: (keys 16jj+0..7, dims lo), (keys 0..7, dims hi), (keys 8..15, lo), (keys 8..15, hi)
-        const int key = jj * 16 + (lane & 7) + ((lane >> 4) << 3);
-        const int ch = kk * 2 + ((lane >> 3) & 1);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(kbase + kv_off<HD>(key, ch), b0, b1, b2, b3);
-        mma_bf16_16816(s[2 * jj], qf[kk], b0, b1);
-        mma_bf16_16816(s[2 * jj + 1], qf[kk], b2, b3);
-      }
-    }
-    // scale, mask, online softmax (base 2)
-    const int kbase_idx = chunk * ATT_PAGE;
-    float mx_a = m_a, mx_b = m_b;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int k0 = kbase_idx + j * 8 + tq * 2;
-      s[j][0] = (k0 < vis_a) ? s[j][0] * scale : -INFINITY;
-      s[j][1] = (k0 + 1 < vis_a) ? s[j][1] * scale : -INFINITY;
-      s[j][2] = (k0 < vis_b) ? s[j][2] * scale : -INFINITY;
-      s[j][3] = (k0 + 1 < vis_b) ? s[j][3] * scale : -INFINITY;
-      mx_a = fmaxf(mx_a, fmaxf(s[j][0], s[j][1]));
-      mx_b = fmaxf(mx_b, fmaxf(s[j][2], s[j][3]));
-    }
-    mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 1));
-    mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 2));
-    mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 1));
-    mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 2));
-    const float ua = (mx_a == -INFINITY) ? 0.f : mx_a;
-    const float ub = (mx_b == -INFINITY) ? 0.f : mx_b;
-    const float alpha_a = exp2f(m_a - ua), alpha_b = exp2f(m_b - ub);
-    m_a = mx_a;
-    m_b = mx_b;
-    l_a *= alpha_a;
-    l_b *= alpha_b;
-#pragma unroll
-    for (int j = 0; j < NDT; ++j) {
-      o[j][0] *= alpha_a;
-      o[j][1] *= alpha_a;
-      o[j][2] *= alpha_b;
-      o[j][3] *= alpha_b;
-    }
-    uint32_t ph[4][4], pl[4][4];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float p0 = exp2f(s[j][0] - ua), p1 = exp2f(s[j][1] - ua);
-      const float p2 = exp2f(s[j][2] - ub), p3 = exp2f(s[j][3] - ub);
-      l_a += p0 + p1;
-      l_b += p2 + p3;
-      const int kk = j >> 1, r = (j & 1) * 2;
-      split_f16(p0, p1, ph[kk][r], pl[kk][r]);
-      split_f16(p2, p3, ph[kk][r + 1], pl[kk][r + 1]);
-    }
-    // O += P V with P = hi + lo (fp16) and V fp16 (exactly the bf16-rounded values)
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-#pragma unroll
-      for (int dd = 0; dd < NDT / 2; ++dd) {
-        // trans matrices: (keys 16kk+0..7, dims 16dd+0..7), (keys +8..15, same), (keys 0..7, dims +8..15), (8..15, +8..15)
-        const int key = kk * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
-        const int ch = dd * 2 + (lane >> 4);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(vbase + kv_off<HD>(key, ch), b0, b1, b2, b3);
-        mma_f16_16816(o[2 * dd], ph[kk], b0, b1);
-        mma_f16_16816(o[2 * dd + 1], ph[kk], b2, b3);
-        mma_f16_16816(o[2 * dd], pl[kk], b0, b1);
-        mma_f16_16816(o[2 * dd + 1], pl[kk], b2, b3);
-      }
-    }
-    __syncthreads();  // buffer `buf` may be refilled next iteration
-  }
-  if (!ok) {
-    // wait (bounded) for any copy still in flight before the CTA exits
-    if (tid == 0) {
-      for (int b = 0; b < 2; ++b) mbar_wait(&bars[b], 0, nullptr), mbar_wait(&bars[b], 1, nullptr);
-    }
-    __syncthreads();
-    return;
-  }
-  l_a += __shfl_xor_sync(0xffffffffu, l_a, 1);
-  l_a += __shfl_xor_sync(0xffffffffu, l_a, 2);
-  l_b += __shfl_xor_sync(0xffffffffu, l_b, 1);
-  l_b += __shfl_xor_sync(0xffffffffu, l_b, 2);
-
-  if (a.direct) {
-    const float ia = l_a > 0.f ? 1.f / l_a : 0.f, ib = l_b > 0.f ? 1.f / l_b : 0.f;
-#pragma unroll
-    for (int j = 0; j < NDT; ++j) {
-      const int col = h * HD + j * 8 + tq * 2;
-      if (row_a < nq)
-        *reinterpret_cast<__nv_bfloat162*>(a.out + (size_t)(t0 + row_a) * d + col) =
-            __floats2bfloat162_rn(o[j][0] * ia, o[j][1] * ia);
-      if (row_b < nq)
-        *reinterpret_cast<__nv_bfloat162*>(a.out + (size_t)(t0 + row_b) * d + col) =
-            __floats2bfloat162_rn(o[j][2] * ib, o[j][3] * ib);
-    }
-  } else {
-    const size_t base = (size_t)split * a.T;
-#pragma unroll
-    for (int j = 0; j < NDT; ++j) {
-      const int col = j * 8 + tq * 2;
-      if (row_a < nq)
-        *reinterpret_cast<float2*>(a.part_o + ((base + t0 + row_a) * a.n_heads + h) * HD + col) =
-            make_float2(o[j][0], o[j][1]);
-      if (row_b < nq)
-        *reinterpret_cast<float2*>(a.part_o + ((base + t0 + row_b) * a.n_heads + h) * HD + col) =
-            make_float2(o[j][2], o[j][3]);
-    }
-    if (tq == 0) {
-      if (row_a < nq)
-        *reinterpret_cast<float2*>(a.part_ml + ((base + t0 + row_a) * a.n_heads + h) * 2) = make_float2(m_a, l_a);
-      if (row_b < nq)
-        *reinterpret_cast<float2*>(a.part_ml + ((base + t0 + row_b) * a.n_heads + h) * 2) = make_float2(m_b, l_b);
-    }
-  }
+  __syncthreads();
+  int use[2] = {0, 0};
+  attn_item<HD>(a, &mk, &mv, blockIdx.x, blockIdx.y, blockIdx.z, smem, bars, s_info, use, threadIdx.x, 1);
 }
 
-// One warp per (token, head): merge the prefix splits with the token's path keys.
+// One CTA of 128 threads per (query tile, head): merge the prefix splits with the path keys.
 template <int HD>
-__global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs a) {
-  constexpr int PER = HD / 32;
+__global__ void __launch_bounds__(128) attn_combine_kernel(const AttnArgs a) {
   pdl_launch_dependents();
   pdl_wait();
-  const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (gw >= a.T * a.n_heads) return;
-  const int t = gw / a.n_heads, h = gw % a.n_heads;
-  const int d = a.n_heads * HD;
-  const int u = a.tok_user[t];
-  const int S = a.user_splits[u];
-  const float scale = kLog2e / sqrtf((float)HD);
-  float qv[PER];
-#pragma unroll
-  for (int i = 0; i < PER; ++i) qv[i] = __bfloat162float(a.q[(size_t)t * d + h * HD + lane + 32 * i]);
-  const int na = a.anc_n ? a.anc_n[t] : 0;
-  float sa[ATT_MAX_ANC];
-  float M = -INFINITY;
-  for (int j = 0; j < na; ++j) {
-    const int row = a.anc_row[t * ATT_MAX_ANC + j];
-    float acc = 0.f;
-#pragma unroll
-    for (int i = 0; i < PER; ++i) acc += qv[i] * __bfloat162float(a.k_cache[(size_t)row * d + h * HD + lane + 32 * i]);
-    acc = warp_sum(acc) * scale;
-    sa[j] = acc;
-    M = fmaxf(M, acc);
-  }
-  for (int s = 0; s < S; ++s) {
-    const float m = a.part_ml[(((size_t)s * a.T + t) * a.n_heads + h) * 2];
-    M = fmaxf(M, m);
-  }
-  const float Mu = (M == -INFINITY) ? 0.f : M;
-  float L = 0.f, o[PER];
-#pragma unroll
-  for (int i = 0; i < PER; ++i) o[i] = 0.f;
-  for (int s = 0; s < S; ++s) {
-    const size_t b = ((size_t)s * a.T + t) * a.n_heads + h;
-    const float m = a.part_ml[b * 2], l = a.part_ml[b * 2 + 1];
-    const float w = exp2f(m - Mu);
-    L += l * w;
-#pragma unroll
-    for (int i = 0; i < PER; ++i) o[i] += a.part_o[b * HD + lane + 32 * i] * w;
-  }
-  for (int j = 0; j < na; ++j) {
-    const int row = a.anc_row[t * ATT_MAX_ANC + j];
-    const float w = exp2f(sa[j] - Mu);
-    L += w;
-#pragma unroll
-    for (int i = 0; i < PER; ++i) o[i] += w * __half2float(a.v_cache[(size_t)row * d + h * HD + lane + 32 * i]);
-  }
-  const float inv = L > 0.f ? 1.f / L : 0.f;
-#pragma unroll
-  for (int i = 0; i < PER; ++i) a.out[(size_t)t * d + h * HD + lane + 32 * i] = __float2bfloat16_rn(o[i] * inv);
+  attn_combine_tile<HD>(a, blockIdx.x, blockIdx.y, threadIdx.x);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn_att() {
@@ -390,9 +79,8 @@ cudaError_t launch_hd(const AttnArgs& a, const CUtensorMap& mk, const CUtensorMa
   cudaError_t e = cudaLaunchKernelEx(&cfg, attn_prefix_kernel<HD>, mk, mv, a);
   if (e != cudaSuccess || a.direct) return e;
   cudaLaunchConfig_t c2 = {};
-  const int warps = a.T * a.n_heads;
-  c2.gridDim = dim3((warps + 7) / 8);
-  c2.blockDim = dim3(256);
+  c2.gridDim = dim3(a.n_qtiles, a.n_heads);
+  c2.blockDim = dim3(128);
   c2.stream = st;
   c2.attrs = at;
   c2.numAttrs = pdl ? 1 : 0;

@@ -1,0 +1,731 @@
+// Persistent forward kernel for sm_103a.
+//
+// One cooperative launch, one CTA per SM, runs a whole decoder forward as a fixed phase program:
+//   NORM0 | for each layer: QKV, ATTN, O, NORM, GATE_UP, DOWN, NORM | LM
+// with a grid barrier after every phase.  The GEMM phases reuse the stream-K decomposition of the
+// standalone GEMM (equal contiguous ranges of (tile, k-block) units per CTA, split tiles reduced
+// by their last CTA), but their operands flow through two rings that live for the whole launch:
+//   * the weight ring (A, 16 KB per stage) is filled by a producer warp that walks every GEMM
+//     phase of the forward in order and never waits for a grid barrier -- weights do not depend
+//     on activations -- so HBM keeps streaming the next phase's weights during barriers, norms
+//     and attention;
+//   * the activation ring (B) is filled by a second producer warp that waits for the barrier that
+//     publishes the phase's input.
+// Warp roles (256 threads): 0 weight TMA, 1 activation TMA, 2 TMEM + MMA issue, 3 idle,
+// 4..7 compute (GEMM epilogues on TMEM lane quadrants 0..3, RMSNorm rows, tree attention).
+// Every wait is bounded; a timeout (or an error raised by another CTA) makes every role leave its
+// loop, in-flight copies are waited for, TMEM is released.
+#include <cudaTypedefs.h>
+#include <stdio.h>
+
+#include "attn_core.cuh"
+#include "common.cuh"
+#include "fwd.cuh"
+#include "gemm_core.cuh"
+#include "norm_core.cuh"
+
+namespace atspeed {
+
+namespace {
+
+constexpr int FWD_THREADS = 256;
+constexpr int COMPUTE_WARP0 = 4;
+constexpr int ITEM_ROWS_FWD = 1024;   // item-code rows of the LM head (4 levels x 256 codes)
+
+template <int BN>
+struct FCfg {
+  static constexpr int SA = BN == 128 ? 6 : 4;   // weight stages
+  static constexpr int SB = BN == 128 ? 5 : 3;   // activation stages
+  static constexpr int A_BYTES = GEMM_BM * 128;
+  static constexpr int B_BYTES = BN * 128;
+  static constexpr int STAGING = 32 * GEMM_BM * 4;
+  static constexpr int MISC = 4096;
+  static constexpr int TMEM_COLS = 2 * BN;
+};
+
+template <int HD, int BN>
+struct FLayout {
+  using C = FCfg<BN>;
+  static constexpr int A_OFF = 0;
+  static constexpr int B_OFF = C::SA * C::A_BYTES;
+  static constexpr int STG_OFF = B_OFF + C::SB * C::B_BYTES;
+  // the attention work area overlaps the activation ring and the staging buffer (both idle then)
+  static constexpr int ATT_OFF = B_OFF;
+  static constexpr int ATT_NEED = AttCfg<HD>::SMEM_BODY;
+  static constexpr int AFTER_STG = STG_OFF + C::STAGING;
+  static constexpr int EXTRA = (ATT_OFF + ATT_NEED > AFTER_STG) ? ((ATT_OFF + ATT_NEED - AFTER_STG + 1023) / 1024) * 1024 : 0;
+  static constexpr int MISC_OFF = AFTER_STG + EXTRA;
+  static constexpr int TOTAL = 1024 + MISC_OFF + C::MISC;
+};
+
+struct GP {
+  int epi;
+  int M, K, m_tiles, n_tiles, kb, up_row0, rows;  // rows: valid tokens of the phase
+  long long U;
+  int Ge;        // CTAs that receive units: min(G, U) (the others idle in this phase)
+  int mapA, mapB, layer;
+};
+
+__device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
+  GP g;
+  const int L = p.L;
+  const int act0 = 6 * L + 1 + (BN == 256 ? 3 : 0);   // activation maps: x, att, act
+  g.layer = gi / 4;
+  g.up_row0 = 0;
+  g.rows = p.T;
+  if (gi == 4 * L) {
+    g.epi = EPI_F32;
+    g.M = ITEM_ROWS_FWD;
+    g.K = p.d;
+    g.mapA = 6 * L;
+    g.mapB = act0;
+    g.rows = p.n_out;
+  } else {
+    const int k = gi % 4;
+    g.mapA = g.layer * 4 + k;
+    if (k == 0) {
+      g.epi = EPI_QKV;
+      g.M = 3 * p.d;
+      g.K = p.d;
+      g.mapB = act0;
+    } else if (k == 1) {
+      g.epi = EPI_RESID;
+      g.M = p.d;
+      g.K = p.d;
+      g.mapB = act0 + 1;
+    } else if (k == 2) {
+      g.epi = EPI_SWIGLU;
+      g.M = 2 * p.ffn;
+      g.K = p.d;
+      g.up_row0 = p.ffn;
+      g.mapB = act0;
+    } else {
+      g.epi = EPI_RESID;
+      g.M = p.d;
+      g.K = p.ffn;
+      g.mapB = act0 + 2;
+    }
+  }
+  g.m_tiles = (g.epi == EPI_SWIGLU) ? g.M / GEMM_BM : (g.M + GEMM_BM - 1) / GEMM_BM;
+  g.n_tiles = (g.rows + BN - 1) / BN;
+  g.kb = g.K / GEMM_BK;
+  g.U = (long long)g.m_tiles * g.n_tiles * g.kb;
+  g.Ge = (int)((long long)p.G < g.U ? p.G : g.U);
+  return g;
+}
+
+// This CTA's unit range [u0, u1) of a GEMM phase (same partition as the standalone GEMM).
+__device__ __forceinline__ void crange(const GP& g, int c, long long& u0, long long& u1) {
+  if (c >= g.Ge) {
+    u0 = u1 = 0;
+    return;
+  }
+  u0 = (long long)c * g.U / g.Ge;
+  u1 = (long long)(c + 1) * g.U / g.Ge;
+}
+
+// phase index (in the compute warps' program) of GEMM phase gi
+__device__ __forceinline__ int gemm_phase_index(int gi, int L) {
+  if (gi == 4 * L) return 1 + 7 * L;
+  const int l = gi / 4, k = gi % 4;
+  return 7 * l + (k == 0 ? 1 : k == 1 ? 3 : k == 2 ? 5 : 6);
+}
+
+__device__ __forceinline__ long long ustart(long long c, long long U, int G) { return c * U / G; }
+__device__ __forceinline__ int uowner(long long u, long long U, int G) { return (int)(((u + 1) * (long long)G - 1) / U); }
+
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* a) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
+__device__ __forceinline__ bool err_set(const unsigned* e) { return *(volatile const unsigned*)e != 0u; }
+
+// Waits until barrier `k` (0-based) is complete: count >= (k + 1) * G.  False on timeout or when an
+// error was raised anywhere.
+__device__ bool grid_wait(const FwdParams& p, int k) {
+  const unsigned target = (unsigned)(k + 1) * (unsigned)p.G;
+  if (ld_acquire_u32(p.bar) >= target) return true;
+  const unsigned long long t0 = globaltimer_ns();
+  for (unsigned it = 1;; ++it) {
+    __nanosleep(64);
+    if (ld_acquire_u32(p.bar) >= target) return true;
+    if ((it & 255u) == 0u) {
+      if (err_set(p.err)) return false;
+      if (globaltimer_ns() - t0 > kWaitBudgetNs) {
+        set_error(p.err, ATSPEED_DEV_ERR_TIMEOUT);
+        return false;
+      }
+    }
+  }
+}
+
+// mbarrier wait that also gives up as soon as an error is raised anywhere
+__device__ bool mwait(uint64_t* bar, uint32_t parity, unsigned* err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = globaltimer_ns();
+  for (unsigned it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 1023u) == 0u) {
+      if (err_set(err)) return false;
+      if (globaltimer_ns() - t0 > kWaitBudgetNs) {
+        set_error(err, ATSPEED_DEV_ERR_TIMEOUT);
+        return false;
+      }
+    }
+  }
+}
+
+template <int BN, int EPI>
+__device__ __forceinline__ void epi_dispatch_t(const GemmArgs& a, const float* st, int mt, int nt, int ch, int t) {
+  epi_chunk<BN, EPI>(a, st, mt, nt, ch, t);
+}
+template <int BN>
+__device__ __forceinline__ void epi_dispatch(int epi, const GemmArgs& a, const float* st, int mt, int nt, int ch,
+                                             int t) {
+  switch (epi) {
+    case EPI_F32: epi_dispatch_t<BN, EPI_F32>(a, st, mt, nt, ch, t); break;
+    case EPI_RESID: epi_dispatch_t<BN, EPI_RESID>(a, st, mt, nt, ch, t); break;
+    case EPI_SWIGLU: epi_dispatch_t<BN, EPI_SWIGLU>(a, st, mt, nt, ch, t); break;
+    default: epi_dispatch_t<BN, EPI_QKV>(a, st, mt, nt, ch, t); break;
+  }
+}
+
+__device__ GemmArgs epi_args(const FwdParams& p, const GP& g) {
+  GemmArgs a = {};
+  a.epi = (EpiKind)g.epi;
+  a.M = g.M;
+  a.K = g.K;
+  a.T = g.rows;
+  a.d_model = p.d;
+  a.head_dim = p.hd;
+  a.pos = p.pos;
+  a.kv_row = p.kv_row;
+  a.rope_cos = p.rope_cos;
+  a.rope_sin = p.rope_sin;
+  a.q_out = p.q;
+  a.k_cache = p.kc + p.layer_elems * g.layer;
+  a.v_cache = p.vc + p.layer_elems * g.layer;
+  if (g.epi == EPI_F32) {
+    a.out_f32 = p.logits;
+    a.ldo = ITEM_ROWS_FWD;
+  } else if (g.epi == EPI_RESID) {
+    a.out_f32 = p.h;
+    a.ldo = p.d;
+  } else if (g.epi == EPI_SWIGLU) {
+    a.out_bf16 = p.act;
+    a.ldo = p.ffn;
+  }
+  return a;
+}
+
+// RMSNorm of rows (128 compute threads, two virtual threads each; the sums are the same, bit for
+// bit, as the 256-thread kernels'): mode 0 = embedding gather + norm (layer 0), 1 = norm of h,
+// 2 = final norm of the selected rows.  A row stays in registers between the two passes.
+constexpr int NORM_MAXC = 8;   // float4 chunks per virtual thread: d <= 8192
+
+__device__ void norm_phase(const FwdParams& p, int mode, const __nv_bfloat16* g, float* red, int ctid) {
+  const int rows = mode == 2 ? p.n_out : p.T;
+  const int d = p.d, nc = d / 4;
+  const int w = ctid >> 5;
+  for (int r = blockIdx.x; r < rows; r += p.G) {
+    const int src = mode == 2 ? p.out_rows[r] : r;
+    float* hr = p.h + (size_t)src * d;
+    float4 v[2][NORM_MAXC];
+    float ss[2] = {0.f, 0.f};
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+#pragma unroll
+      for (int k = 0; k < NORM_MAXC; ++k) {
+        const int c = ctid + 128 * s + 256 * k;
+        if (c < nc) {
+          if (mode == 0) {
+            const uint2 raw = *reinterpret_cast<const uint2*>(p.embed + (size_t)p.tok[r] * d + 4 * c);
+            const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&raw);
+            const float2 f0 = __bfloat1622float2(b[0]), f1 = __bfloat1622float2(b[1]);
+            v[s][k] = make_float4(f0.x, f0.y, f1.x, f1.y);
+            *reinterpret_cast<float4*>(hr + 4 * c) = v[s][k];
+          } else {
+            v[s][k] = __ldcg(reinterpret_cast<const float4*>(hr) + c);
+          }
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < NORM_MAXC; ++k) {
+        const int c = ctid + 128 * s + 256 * k;
+        if (c < nc) {
+          ss[s] += v[s][k].x * v[s][k].x;
+          ss[s] += v[s][k].y * v[s][k].y;
+          ss[s] += v[s][k].z * v[s][k].z;
+          ss[s] += v[s][k].w * v[s][k].w;
+        }
+      }
+    }
+    const float sa = warp_sum(ss[0]), sb = warp_sum(ss[1]);
+    if ((ctid & 31) == 0) {
+      red[w] = sa;
+      red[w + 4] = sb;
+    }
+    named_bar_sync(1, 128);
+    const float rs = 1.0f / sqrtf(rms_total(red) / (float)d + p.eps);
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+#pragma unroll
+      for (int k = 0; k < NORM_MAXC; ++k) {
+        const int c = ctid + 128 * s + 256 * k;
+        if (c < nc) {
+          const uint2 graw = *reinterpret_cast<const uint2*>(g + 4 * c);
+          const __nv_bfloat162* gb = reinterpret_cast<const __nv_bfloat162*>(&graw);
+          const float2 g0 = __bfloat1622float2(gb[0]), g1 = __bfloat1622float2(gb[1]);
+          __nv_bfloat162 o[2];
+          o[0] = __floats2bfloat162_rn(v[s][k].x * rs * g0.x, v[s][k].y * rs * g0.y);
+          o[1] = __floats2bfloat162_rn(v[s][k].z * rs * g1.x, v[s][k].w * rs * g1.y);
+          *reinterpret_cast<uint2*>(p.x + (size_t)r * d + 4 * c) = *reinterpret_cast<uint2*>(o);
+        }
+      }
+    }
+    named_bar_sync(1, 128);
+  }
+}
+
+template <int HD, int BN>
+__global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) {
+  using C = FCfg<BN>;
+  using LY = FLayout<HD, BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* ringA = smem + LY::A_OFF;
+  uint8_t* ringB = smem + LY::B_OFF;
+  float* staging = reinterpret_cast<float*>(smem + LY::STG_OFF);
+  uint8_t* att_smem = smem + LY::ATT_OFF;
+  uint64_t* fullA = reinterpret_cast<uint64_t*>(smem + LY::MISC_OFF);
+  uint64_t* emptyA = fullA + C::SA;
+  uint64_t* fullB = emptyA + C::SA;
+  uint64_t* emptyB = fullB + C::SB;
+  uint64_t* tfull = emptyB + C::SB;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* mma_done = tempty + 2;
+  uint64_t* att_bars = mma_done + 1;                              // 2
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(att_bars + 2);
+  int* flag = reinterpret_cast<int*>(tmem_slot + 1);
+  int* failed = flag + 1;
+  int* lastA = failed + 1;                                        // [SA] parity of last fill, -1 none
+  int* lastB = lastA + C::SA;                                     // [SB]
+  int* s_info = lastB + C::SB;                                    // 2 (attention)
+  float* red = reinterpret_cast<float*>(s_info + 2);              // 8
+  int* part_slot = reinterpret_cast<int*>(red + 8);               // 256
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = blockIdx.x, G = p.G, L = p.L;
+  const int NG = 4 * L + 1;      // GEMM phases
+  const int NP = 7 * L + 2;      // all phases
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::SA; ++s) {
+      mbar_init(&fullA[s], 1);
+      mbar_init(&emptyA[s], 1);
+      lastA[s] = -1;
+    }
+    for (int s = 0; s < C::SB; ++s) {
+      mbar_init(&fullB[s], 1);
+      mbar_init(&emptyB[s], 1);
+      lastB[s] = -1;
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 4);
+      mbar_init(&att_bars[i], 1);
+    }
+    mbar_init(mma_done, 1);
+    *failed = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------- weight producer (never waits for the grid)
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_first();
+      long long n = 0;
+      bool ok = true;
+      for (int gi = 0; gi < NG && ok; ++gi) {
+        const GP g = gemm_phase(p, gi, BN);
+        const CUtensorMap* mA = p.maps + g.mapA;
+        long long u0, u1;
+        crange(g, c, u0, u1);
+        for (long long u = u0; u < u1; ++u, ++n) {
+          const int s = (int)(n % C::SA);
+          const uint32_t ph = (uint32_t)((n / C::SA) & 1);
+          if (!mwait(&emptyA[s], ph ^ 1u, p.err)) {
+            ok = false;
+            break;
+          }
+          const int tile = (int)(u / g.kb), kbi = (int)(u % g.kb);
+          const int mt = tile / g.n_tiles;
+          int r0, r1;
+          if (g.epi == EPI_SWIGLU) {
+            r0 = mt * 64;
+            r1 = g.up_row0 + mt * 64;
+          } else {
+            r0 = mt * GEMM_BM;
+            r1 = mt * GEMM_BM + 64;
+          }
+          uint8_t* sa = ringA + s * C::A_BYTES;
+          mbar_arrive_expect_tx(&fullA[s], C::A_BYTES);
+          lastA[s] = (int)ph;
+          tma_load_2d(sa, mA, &fullA[s], kbi * GEMM_BK, r0, pol);
+          tma_load_2d(sa + 8192, mA, &fullA[s], kbi * GEMM_BK, r1, pol);
+        }
+      }
+      if (!ok) *failed = 1;
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------- activation producer
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_last();
+      long long n = 0;
+      bool ok = true;
+      for (int gi = 0; gi < NG && ok; ++gi) {
+        const GP g = gemm_phase(p, gi, BN);
+        long long u0, u1;
+        crange(g, c, u0, u1);
+        if (u1 <= u0) continue;
+        if (!grid_wait(p, gemm_phase_index(gi, L) - 1)) {
+          ok = false;
+          break;
+        }
+        if (p.trace) p.trace[((size_t)1 * (7 * L + 2) + gi) * G + c] = globaltimer_ns();
+        fence_proxy_async();
+        const CUtensorMap* mB = p.maps + g.mapB;
+        for (long long u = u0; u < u1; ++u, ++n) {
+          const int s = (int)(n % C::SB);
+          const uint32_t ph = (uint32_t)((n / C::SB) & 1);
+          if (!mwait(&emptyB[s], ph ^ 1u, p.err)) {
+            ok = false;
+            break;
+          }
+          const int tile = (int)(u / g.kb), kbi = (int)(u % g.kb);
+          const int nt = tile % g.n_tiles;
+          mbar_arrive_expect_tx(&fullB[s], C::B_BYTES);
+          lastB[s] = (int)ph;
+          tma_load_2d(ringB + s * C::B_BYTES, mB, &fullB[s], kbi * GEMM_BK, nt * BN, pol);
+        }
+        if (p.trace) p.trace[((size_t)2 * (7 * L + 2) + gi) * G + c] = globaltimer_ns();
+      }
+      if (!ok) *failed = 1;
+    }
+  } else if (warp == 2) {
+    // ------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(GEMM_BM, BN);
+      long long n = 0;
+      int si = 0;
+      int mma_waits = 0;
+      bool ok = true;
+      for (int gi = 0; gi < NG && ok; ++gi) {
+        const GP g = gemm_phase(p, gi, BN);
+        long long u0, u1;
+        crange(g, c, u0, u1);
+        for (long long u = u0; u < u1 && ok; ++si) {
+          const int k0 = (int)(u % g.kb);
+          const long long len = (g.kb - k0) < (u1 - u) ? (g.kb - k0) : (u1 - u);
+          u += len;
+          const int acc = si & 1, use = si >> 1;
+          if (!mwait(&tempty[acc], (uint32_t)(use & 1) ^ 1u, p.err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t dt = tmem_base + (uint32_t)(acc * BN);
+          for (long long j = 0; j < len; ++j, ++n) {
+            const int sa = (int)(n % C::SA), sb = (int)(n % C::SB);
+            const uint32_t pa = (uint32_t)((n / C::SA) & 1), pb = (uint32_t)((n / C::SB) & 1);
+            if (!mwait(&fullA[sa], pa, p.err) || !mwait(&fullB[sb], pb, p.err)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint64_t ad = smem_desc_sw128(smem_u32(ringA + sa * C::A_BYTES));
+            const uint64_t bd = smem_desc_sw128(smem_u32(ringB + sb * C::B_BYTES));
+#pragma unroll
+            for (int kk = 0; kk < GEMM_BK / 16; ++kk)
+              tc_mma_bf16(dt, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), idesc, (j > 0 || kk > 0) ? 1u : 0u);
+            tc_commit(&emptyA[sa]);
+            tc_commit(&emptyB[sb]);
+          }
+          if (!ok) break;
+          tc_commit(&tfull[acc]);
+        }
+        if (p.trace && u1 > u0) {
+          // time the last MMA of this phase completed
+          tc_commit(mma_done);
+          mbar_wait(mma_done, (uint32_t)(mma_waits & 1), nullptr);
+          ++mma_waits;
+          p.trace[((size_t)3 * (7 * L + 2) + gi) * G + c] = globaltimer_ns();
+        }
+      }
+      if (!ok) *failed = 1;
+      tc_commit(mma_done);
+      mbar_wait(mma_done, (uint32_t)(mma_waits & 1), nullptr);
+    }
+  } else if (warp >= COMPUTE_WARP0) {
+    // ------------------------------------------------------------- compute warps
+    const int ctid = threadIdx.x - COMPUTE_WARP0 * 32;
+    const int q = warp & 3;      // TMEM lane quadrant
+    const int m = q * 32 + lane;
+    int si = 0;
+    int use_att[2] = {0, 0};
+    bool ok = true;
+    for (int ph = 0; ph < NP && ok; ++ph) {
+      // which phase is this?
+      int kind, l = 0;   // 0 NORM0, 1 GEMM, 2 ATTN, 3 NORM (mlp), 4 NORM (next attn / final)
+      int gi = -1;
+      if (ph == 0) {
+        kind = 0;
+      } else if (ph == NP - 1) {
+        kind = 1;
+        gi = 4 * L;
+      } else {
+        l = (ph - 1) / 7;
+        const int r = (ph - 1) % 7;
+        if (r == 0 || r == 2 || r == 4 || r == 5) {
+          kind = 1;
+          gi = 4 * l + (r == 0 ? 0 : r == 2 ? 1 : r == 4 ? 2 : 3);
+        } else if (r == 1) {
+          kind = 2;
+        } else if (r == 3) {
+          kind = 3;
+        } else {
+          kind = 4;
+        }
+      }
+      if (ph > 0) {
+        // Barrier ph-1 must be complete before this CTA can arrive at barrier ph: the arrival counter
+        // is shared by all barriers, so an early arrival would count towards the previous one.
+        // (Non-GEMM phases also read what the previous phase wrote.)
+        if (ctid == 0) *flag = grid_wait(p, ph - 1) ? 1 : 0;
+        named_bar_sync(1, 128);
+        if (!*flag) {
+          ok = false;
+          break;
+        }
+        fence_proxy_async();
+        named_bar_sync(1, 128);
+      }
+      if (kind == 0) {
+        norm_phase(p, 0, p.attn_norm[0], red, ctid);
+      } else if (kind == 3) {
+        norm_phase(p, 1, p.mlp_norm[l], red, ctid);
+      } else if (kind == 4) {
+        if (l + 1 < L)
+          norm_phase(p, 1, p.attn_norm[l + 1], red, ctid);
+        else
+          norm_phase(p, 2, p.final_norm, red, ctid);
+      } else if (kind == 2) {
+        AttnArgs a = p.att_args;
+        a.k_cache = p.kc + p.layer_elems * l;
+        a.v_cache = p.vc + p.layer_elems * l;
+        const CUtensorMap* mk = p.maps + 4 * L + 2 * l;
+        const CUtensorMap* mv = mk + 1;
+        const int H = p.H, S = a.max_splits;
+        for (int item = c; item < p.att_items && ok; item += G) {
+          const int tile = item / (H * S), rem = item % (H * S);
+          const int h = rem / S, split = rem % S;
+          if (!attn_item<HD>(a, mk, mv, tile, h, split, att_smem, att_bars, s_info, use_att, ctid, 1)) {
+            ok = false;
+            break;
+          }
+          if (a.direct) continue;
+          const int S_u = a.user_splits[a.qt_user[tile]];
+          if (split >= S_u) continue;
+          __threadfence();
+          named_bar_sync(1, 128);
+          if (ctid == 0) {
+            const int old = atomicAdd(&p.att_counters[tile * H + h], 1);
+            const int last = old == S_u - 1;
+            if (last) {
+              p.att_counters[tile * H + h] = 0;
+              __threadfence();
+            }
+            *flag = last;
+          }
+          named_bar_sync(1, 128);
+          if (*flag) attn_combine_tile<HD>(a, tile, h, ctid);
+          named_bar_sync(1, 128);
+        }
+      } else {
+        // ---- GEMM epilogue for this CTA's segments of phase gi
+        const GP g = gemm_phase(p, gi, BN);
+        const GemmArgs ea = epi_args(p, g);
+        const int kb = g.kb;
+        long long u0, u1;
+        crange(g, c, u0, u1);
+        int seg = 0;
+        for (long long u = u0; u < u1 && ok; ++si, ++seg) {
+          const int tile = (int)(u / kb);
+          const int k0 = (int)(u % kb);
+          const long long len = (kb - k0) < (u1 - u) ? (kb - k0) : (u1 - u);
+          const int k1 = k0 + (int)len;
+          u += len;
+          const int acc = si & 1, use = si >> 1;
+          const bool got = mwait(&tfull[acc], (uint32_t)(use & 1), p.err);
+          __syncwarp();
+          if (!got) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const int m_tile = tile / g.n_tiles, n_tile = tile % g.n_tiles;
+          const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+          const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
+          if (k0 == 0 && k1 == kb) {
+            for (int ch = 0; ch < nch; ++ch) {
+              uint32_t r[32];
+              tmem_ld_32x32b_x32(tb + ch * 32, r);
+              tmem_ld_wait();
+#pragma unroll
+              for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = __uint_as_float(r[j]);
+              named_bar_sync(1, 128);
+              epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid);
+              named_bar_sync(1, 128);
+            }
+            tc_fence_before();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+          } else {
+            const long long slot = (long long)c * 2 + (seg == 0 ? 0 : 1);
+            float* wsl = p.ws + slot * GEMM_WS_SLOT_FLOATS;
+            for (int ch = 0; ch < nch; ++ch) {
+              uint32_t r[32];
+              tmem_ld_32x32b_x32(tb + ch * 32, r);
+              tmem_ld_wait();
+#pragma unroll
+              for (int j = 0; j < 32; ++j) __stcg(&wsl[(ch * 32 + j) * GEMM_BM + m], __uint_as_float(r[j]));
+            }
+            tc_fence_before();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+            __threadfence();
+            named_bar_sync(1, 128);
+            const long long tu0 = (long long)tile * kb;
+            const int c_first = uowner(tu0, g.U, g.Ge);
+            const int c_last = uowner(tu0 + kb - 1, g.U, g.Ge);
+            const int parts = c_last - c_first + 1;
+            if (ctid == 0) {
+              const int old = atomicAdd(&p.counters[tile], 1);
+              const int last = (old == parts - 1);
+              if (last) {
+                p.counters[tile] = 0;
+                __threadfence();
+              }
+              *flag = last;
+            }
+            for (int pi = ctid; pi < parts; pi += 128) {
+              const int cc = c_first + pi;
+              part_slot[pi] = cc * 2 + (ustart(cc, g.U, g.Ge) >= tu0 ? 0 : 1);
+            }
+            named_bar_sync(1, 128);
+            if (*flag) {
+              for (int ch = 0; ch < nch; ++ch) {
+                float accv[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) accv[j] = 0.f;
+                for (int pi = 0; pi < parts; ++pi) {
+                  const float* src = p.ws + (long long)part_slot[pi] * GEMM_WS_SLOT_FLOATS + (ch * 32) * GEMM_BM + m;
+                  float v[32];
+#pragma unroll
+                  for (int j = 0; j < 32; ++j) v[j] = __ldcg(src + j * GEMM_BM);
+#pragma unroll
+                  for (int j = 0; j < 32; ++j) accv[j] += v[j];
+                }
+#pragma unroll
+                for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = accv[j];
+                named_bar_sync(1, 128);
+                epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid);
+                named_bar_sync(1, 128);
+              }
+            }
+            named_bar_sync(1, 128);  // flag and part_slot are reused by the next segment
+          }
+        }
+        if (!ok) break;
+      }
+      if (p.trace && ctid == 0) p.trace[(size_t)ph * G + c] = globaltimer_ns();
+      // publish this phase: this CTA's generic-proxy stores must be visible to the other CTAs'
+      // TMA (async-proxy) reads of the next phases, hence the proxy fence before the release
+      if (ph < NP - 1) {
+        fence_proxy_async();
+        __threadfence();
+        named_bar_sync(1, 128);
+        if (ctid == 0) atomicAdd(p.bar, 1u);
+      }
+    }
+    if (!ok) *failed = 1;
+  }
+
+  __syncthreads();
+  if (*failed && threadIdx.x == 0) {
+    set_error(p.err, ATSPEED_DEV_ERR_TIMEOUT);
+    for (int s = 0; s < C::SA; ++s)
+      if (lastA[s] >= 0) mbar_wait(&fullA[s], (uint32_t)lastA[s], nullptr);
+    for (int s = 0; s < C::SB; ++s)
+      if (lastB[s] >= 0) mbar_wait(&fullB[s], (uint32_t)lastB[s], nullptr);
+  }
+  __syncthreads();
+  if (warp == 2) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+template <int HD, int BN>
+cudaError_t launch_t(const FwdParams& p, cudaStream_t st) {
+  using LY = FLayout<HD, BN>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(fwd_kernel<HD, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, LY::TOTAL);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.G);
+  cfg.blockDim = dim3(FWD_THREADS);
+  cfg.dynamicSmemBytes = LY::TOTAL;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeCooperative;
+  at[0].val.cooperative = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, fwd_kernel<HD, BN>, p);
+}
+
+template <int HD>
+cudaError_t launch_hd(const FwdParams& p, cudaStream_t st) {
+  return p.T <= 128 ? launch_t<HD, 128>(p, st) : launch_t<HD, 256>(p, st);
+}
+
+}  // namespace
+
+size_t fwd_smem_bytes(int hd, int bn) {
+  if (bn == 128) return hd == 32 ? FLayout<32, 128>::TOTAL : hd == 64 ? FLayout<64, 128>::TOTAL : FLayout<128, 128>::TOTAL;
+  return hd == 32 ? FLayout<32, 256>::TOTAL : hd == 64 ? FLayout<64, 256>::TOTAL : FLayout<128, 256>::TOTAL;
+}
+
+cudaError_t fwd_launch(const FwdParams& p, cudaStream_t st) {
+  switch (p.hd) {
+    case 32: return launch_hd<32>(p, st);
+    case 64: return launch_hd<64>(p, st);
+    case 128: return launch_hd<128>(p, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace atspeed

@@ -18,6 +18,7 @@
 
 #include "common.cuh"
 #include "gemm.cuh"
+#include "gemm_core.cuh"
 
 namespace atspeed {
 
@@ -54,65 +55,6 @@ struct KParams {
 __device__ __forceinline__ long long unit_start(long long c, long long U, int G) { return c * U / G; }
 __device__ __forceinline__ int unit_owner(long long u, long long U, int G) {
   return (int)(((u + 1) * (long long)G - 1) / U);
-}
-
-template <int BN, int EPI>
-__device__ __forceinline__ void epi_chunk(const KParams& p, const float* st, int m_tile, int n_tile, int ch,
-                                          int ep_tid) {
-  const GemmArgs& a = p.a;
-  const int tok0 = n_tile * BN + ch * 32;
-  if constexpr (EPI == EPI_SWIGLU) {
-    for (int idx = ep_tid; idx < 32 * 64; idx += 128) {
-      const int n = idx >> 6, i = idx & 63;
-      const int tok = tok0 + n;
-      if (tok >= a.T) continue;
-      const float g = st[n * BM + i];
-      const float u = st[n * BM + 64 + i];
-      const float s = g / (1.0f + expf(-g));
-      a.out_bf16[(size_t)tok * a.ldo + m_tile * 64 + i] = __float2bfloat16_rn(s * u);
-    }
-  } else {
-    for (int idx = ep_tid; idx < 32 * BM; idx += 128) {
-      const int n = idx >> 7, m = idx & 127;
-      const int tok = tok0 + n;
-      const int row = m_tile * BM + m;
-      if (tok >= a.T || row >= a.M) continue;
-      const float v = st[idx];
-      if constexpr (EPI == EPI_F32) {
-        a.out_f32[(size_t)tok * a.ldo + row] = v;
-      } else if constexpr (EPI == EPI_BF16) {
-        a.out_bf16[(size_t)tok * a.ldo + row] = __float2bfloat16_rn(v);
-      } else if constexpr (EPI == EPI_RESID) {
-        float* o = a.out_f32 + (size_t)tok * a.ldo + row;
-        *o = *o + v;
-      } else {  // EPI_QKV
-        const int d = a.d_model, hd = a.head_dim, half = hd >> 1;
-        const int region = row / d;
-        const int f = row - region * d;
-        if (region == 2) {
-          a.v_cache[(size_t)a.kv_row[tok] * d + f] = __float2half_rn(bf16_round(v));
-        } else {
-          const int i = f % hd;
-          const int ii = (i < half) ? i : i - half;
-          const size_t cs = (size_t)a.pos[tok] * half + ii;
-          const float cth = a.rope_cos[cs], sth = a.rope_sin[cs];
-          float out;
-          if (i < half) {
-            const float x2 = st[n * BM + m + half];
-            out = v * cth - x2 * sth;
-          } else {
-            const float x1 = st[n * BM + m - half];
-            out = v * cth + x1 * sth;
-          }
-          const __nv_bfloat16 ob = __float2bfloat16_rn(out);
-          if (region == 0)
-            a.q_out[(size_t)tok * d + f] = ob;
-          else
-            a.k_cache[(size_t)a.kv_row[tok] * d + f] = ob;
-        }
-      }
-    }
-  }
 }
 
 template <int BN, int EPI>
@@ -302,7 +244,7 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
           for (int j = 0; j < 32; ++j) staging[j * BM + m] = __uint_as_float(r[j]);
           named_bar_sync(1, 128);
-          epi_chunk<BN, EPI>(p, staging, m_tile, n_tile, ch, ep_tid);
+          epi_chunk<BN, EPI>(p.a, staging, m_tile, n_tile, ch, ep_tid);
           named_bar_sync(1, 128);
         }
         tc_fence_before();
@@ -356,7 +298,7 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
             for (int j = 0; j < 32; ++j) staging[j * BM + m] = accv[j];
             named_bar_sync(1, 128);
-            epi_chunk<BN, EPI>(p, staging, m_tile, n_tile, ch, ep_tid);
+            epi_chunk<BN, EPI>(p.a, staging, m_tile, n_tile, ch, ep_tid);
             named_bar_sync(1, 128);
           }
         }
@@ -448,6 +390,10 @@ cudaError_t launch_bn(EpiKind e, const CUtensorMap& ma, const CUtensorMap& mb, c
 }
 
 }  // namespace
+
+bool gemm_make_map(CUtensorMap* m, const void* base, int inner, int rows, int box_rows, char* eb, size_t el) {
+  return make_map(m, base, inner, rows, box_rows, eb, el);
+}
 
 size_t gemm_ws_bytes(int grid) { return (size_t)2 * grid * WS_SLOT_FLOATS * sizeof(float); }
 int gemm_max_tiles() { return MAX_TILES; }

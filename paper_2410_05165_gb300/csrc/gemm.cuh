@@ -51,6 +51,9 @@ int gemm_max_tiles();
 // Number of CTAs of the persistent stream-K grid (one per SM).
 int gemm_grid_size(int device);
 
+// 2D bf16 tensor map over a row-major [rows][inner] matrix, box {64, box_rows}, 128B swizzle.
+bool gemm_make_map(CUtensorMap* m, const void* base, int inner, int rows, int box_rows, char* eb, size_t el);
+
 // Encodes the tensor maps and launches.  `pdl` enables programmatic dependent launch.
 cudaError_t gemm_launch(const GemmArgs& a, const GemmScratch& s, int grid, cudaStream_t stream, bool pdl,
                         char* errbuf, size_t errlen);

@@ -3,6 +3,7 @@
 //   x[t] = bf16( h[t] / sqrt(mean(h[t]^2) + eps) * g )
 #include "common.cuh"
 #include "kernels.cuh"
+#include "norm_core.cuh"
 
 namespace atspeed {
 
@@ -14,32 +15,12 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ 
   pdl_wait();
   const int t = blockIdx.x;
   __shared__ float red[8];
-  float ss = 0.f;
-  if (tokens) {
-    const __nv_bfloat16* er = embed + (size_t)tokens[t] * d;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) {
-      const float v = __bfloat162float(er[i]);
-      h_out[(size_t)t * d + i] = v;
-      ss += v * v;
-    }
-  } else {
-    const float* hr = h + (size_t)t * d;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) {
-      const float v = hr[i];
-      ss += v * v;
-    }
-  }
+  float* hr = tokens ? h_out + (size_t)t * d : const_cast<float*>(h) + (size_t)t * d;
+  float ss = tokens ? rms_part_embed(embed + (size_t)tokens[t] * d, hr, threadIdx.x, d) : rms_part(hr, threadIdx.x, d);
   ss = warp_sum(ss);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();
-  if (threadIdx.x < 32) {
-    float v = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
-    v = warp_sum(v);
-    if (threadIdx.x == 0) red[0] = v;
-  }
-  __syncthreads();
-  const float r = 1.0f / sqrtf(red[0] / (float)d + eps);
-  const float* hr = tokens ? h_out + (size_t)t * d : h + (size_t)t * d;
+  const float r = 1.0f / sqrtf(rms_total(red) / (float)d + eps);
   for (int i = threadIdx.x; i < d; i += blockDim.x)
     x[(size_t)t * ldx + i] = __float2bfloat16_rn(hr[i] * r * __bfloat162float(g[i]));
 }

@@ -2,6 +2,7 @@
 // final RMSNorm over the rows whose logits are needed.
 #include "common.cuh"
 #include "kernels.cuh"
+#include "norm_core.cuh"
 
 namespace atspeed {
 
@@ -62,18 +63,10 @@ __global__ void __launch_bounds__(256) rmsnorm_rows_kernel(const float* __restri
   __shared__ float red[8];
   const int i = blockIdx.x;
   const float* hr = h + (size_t)rows[i] * d;
-  float ss = 0.f;
-  for (int k = threadIdx.x; k < d; k += blockDim.x) ss += hr[k] * hr[k];
-  ss = warp_sum(ss);
+  float ss = warp_sum(rms_part(hr, threadIdx.x, d));
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();
-  if (threadIdx.x < 32) {
-    float v = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
-    v = warp_sum(v);
-    if (threadIdx.x == 0) red[0] = v;
-  }
-  __syncthreads();
-  const float r = 1.0f / sqrtf(red[0] / (float)d + eps);
+  const float r = 1.0f / sqrtf(rms_total(red) / (float)d + eps);
   for (int k = threadIdx.x; k < d; k += blockDim.x)
     x[(size_t)i * ldx + k] = __float2bfloat16_rn(hr[k] * r * __bfloat162float(g[k]));
 }

@@ -248,3 +248,33 @@ def test_sd_strict_lossless_and_matches_oracle_tiny(ats):
             gaps = np.abs(np.diff(ref_sc.astype(np.float64)))
             assert gaps.min() < 2e-2, (got, ref)
     ctx.close()
+
+
+@pytest.mark.parametrize("cfg,layers", [("tiny", None), ("mid", 2)])
+def test_persistent_forward_equals_per_op_kernels(ats, cfg, layers, monkeypatch):
+    """The persistent forward kernel and the one-kernel-per-op schedule run the same arithmetic in
+    the same order (same stream-K partition, same attention split merge): identical logits, bit for
+    bit, for the prefill rows and for every node of a seeded tree."""
+    w = synth.workload(cfg)
+    spec = w.target if layers is None else synth.ModelSpec(layers, w.target.d_model, w.target.n_heads,
+                                                          w.target.d_ffn, w.target.vocab)
+    items = synth.make_items(min(w.n_items, 5000), w.code_dist, w.zipf_a, w.seed)
+    prompt = synth.make_prompts(1, w.prompt_len, spec.vocab, w.seed)[0]
+    K, N, G = w.K, w.N, 3
+    incoming, levels = synth.random_tree(items, 0, 1, G, N, seed=7)
+    cnt, par, cod, sq = _tree_arrays(levels, 1, G, N)
+    outs = []
+    for mode in ("per_op", "persistent"):
+        monkeypatch.setenv("ATSPEED_FORWARD", mode)
+        ctx = _ctx(ats, spec, None, items, w.code_base, 1, len(prompt), K, N, G, seed=w.seed)
+        _prefill(ats, ctx, [prompt])
+        o = ats.opts(K, N, G)
+        ctx.begin_step(o)
+        ctx.set_tree(cnt, par, cod, sq)
+        root = ctx.node_logits(0, 0, 0)
+        ctx.verify(o, ats.STRICT)
+        nodes = [ctx.node_logits(0, 0, K + j * N + k) for j, lvl in enumerate(levels) for k in range(len(lvl))]
+        outs.append((root, np.stack(nodes)))
+        ctx.close()
+    np.testing.assert_array_equal(outs[0][0], outs[1][0])
+    np.testing.assert_array_equal(outs[0][1], outs[1][1])
