@@ -51,6 +51,7 @@ struct ModelRt {
   // activations
   int Tcap = 0, Xrows = 0;
   float* h = nullptr;
+  float* dh = nullptr;   // persistent forward: product of the last O / down projection
   bf16 *x = nullptr, *q = nullptr, *att = nullptr, *act = nullptr;
   float* logits = nullptr;  // [logit_rows][1024]
   int logit_rows = 0;
@@ -281,6 +282,7 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.Tcap = std::max(L.max_users * L.max_prompt, L.max_users * stride);
   m.Xrows = ((m.Tcap + 255) / 256) * 256;
   m.h = dalloc<float>(c, (size_t)m.Tcap * m.d);
+  m.dh = dalloc<float>(c, (size_t)m.Tcap * m.d);
   m.x = dalloc<bf16>(c, (size_t)m.Xrows * m.d);
   m.q = dalloc<bf16>(c, (size_t)m.Tcap * m.d);
   m.att = dalloc<bf16>(c, (size_t)m.Xrows * m.d);
@@ -539,6 +541,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     f.final_norm = m.final_norm;
     f.embed = m.embed;
     f.h = m.h;
+    f.dh = m.dh;
     f.x = m.x;
     f.q = m.q;
     f.att = m.att;
@@ -585,6 +588,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     f.err = c->err_word;
     f.trace = c->fwd_trace;
     CK(cudaMemsetAsync(c->fwd_bar, 0, sizeof(unsigned int), st));
+    if (c->fwd_trace) CK(cudaMemsetAsync(c->fwd_trace, 0, c->fwd_trace_n * sizeof(unsigned long long), st));
     const double wbytes = 2.0 * m.layers * (4.0 * m.d * m.d + 3.0 * m.d * m.ffn) + 2.0 * ITEM_ROWS * m.d;
     ProfScope ps(c, st, 6, wbytes, 2.0 * T * (wbytes / 2.0));
     CK(fwd_launch(f, st));
@@ -1208,7 +1212,7 @@ atspeed_status atspeed_create(const atspeed_model_desc* target, const atspeed_mo
       const char* tr = getenv("ATSPEED_FWD_TRACE");
       if (tr && tr[0] == '1') {
         const int Lmax = std::max(c->tgt.layers, c->drf.present ? c->drf.layers : 0);
-        c->fwd_trace_n = (size_t)4 * (7 * Lmax + 2) * c->fwd_grid;
+        c->fwd_trace_n = (size_t)16 * (7 * Lmax + 2) * c->fwd_grid;
         c->fwd_trace = dalloc<unsigned long long>(c, c->fwd_trace_n);
       }
     }

@@ -35,14 +35,6 @@ __device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
-// p = hi + lo with hi = fp16(p) and lo = fp16(p - hi): 22 significant bits for the P V product.
-__device__ __forceinline__ void split_f16(float p0, float p1, uint32_t& hi, uint32_t& lo) {
-  const __half2 h = __floats2half2_rn(p0, p1);
-  const float2 hf = __half22float2(h);
-  const __half2 l = __floats2half2_rn(p0 - hf.x, p1 - hf.y);
-  hi = *reinterpret_cast<const uint32_t*>(&h);
-  lo = *reinterpret_cast<const uint32_t*>(&l);
-}
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -79,7 +71,9 @@ struct AttCfg {
 // a bounded wait timed out.
 template <int HD>
 __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtensorMap* mv, int tile, int h, int split,
-                          uint8_t* smem, uint64_t* bars, int* s_info, int (&use)[2], int tid, int bar_id) {
+                          uint8_t* smem, uint64_t* bars, int* s_info, int (&use)[2], int tid, int bar_id,
+                          unsigned long long* tr = nullptr, size_t trs = 0) {
+#define ATT_TR(k) do { if (tr && tid == 0) tr[(size_t)(k) * trs] = globaltimer_ns(); } while (0)
   using C = AttCfg<HD>;
   constexpr int NDT = HD / 8;    // dim n-tiles of O
   constexpr int NKS = HD / 16;   // k-steps of Q K^T
@@ -93,33 +87,24 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
   const int S_u = a.user_splits[u];
   if (split >= S_u) return true;
 
-  if (tid == 0) {
+  // longest visible prefix of the tile's queries (one load per thread, then a max over the CTA)
+  {
     int mv_ = 0;
-    for (int i = 0; i < nq; ++i) mv_ = max(mv_, a.tok_vis[t0 + i]);
-    const int nch = (mv_ + ATT_PAGE - 1) / ATT_PAGE;
-    int c0 = 0, c1 = nch;
-    if (a.chunks_per_split > 0) {
-      c0 = min(nch, split * a.chunks_per_split);
-      c1 = min(nch, c0 + a.chunks_per_split);
-    }
-    s_info[0] = c0;
-    s_info[1] = c1;
-  }
-  // Q tile -> shared memory (rows >= nq are zero)
-  for (int i = tid; i < ATT_QTILE * (HD / 8); i += 128) {
-    const int r = i / (HD / 8), c = i % (HD / 8);
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (r < nq) v = __ldcg(reinterpret_cast<const uint4*>(a.q + (size_t)(t0 + r) * d + h * HD + c * 8));
-    *reinterpret_cast<uint4*>(qs + r * C::QSTRIDE + c * 8) = v;
+    if (tid < nq) mv_ = a.tok_vis[t0 + tid];
+    if (tid + 128 < nq) mv_ = max(mv_, a.tok_vis[t0 + tid + 128]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mv_ = max(mv_, __shfl_xor_sync(0xffffffffu, mv_, o));
+    if (lane == 0) s_info[2 + warp] = mv_;
   }
   named_bar_sync(bar_id, 128);
-  const int c0 = s_info[0], c1 = s_info[1];
+  ATT_TR(0);
   const int* ptab = a.page_table + (size_t)u * a.max_pages;
   constexpr int NBOX = HD >= 64 ? HD / 64 : 1;
   constexpr int BOXW = HD >= 64 ? 64 : HD;
-
+  int c0 = 0, c1 = 0;   // this item's prefix chunks: thread 0 computes them, the others read s_info
+  int page1 = 0;        // page of the second chunk, loaded together with the first one's (thread 0)
   auto issue = [&](int chunk, int buf) {
-    const int row0 = ptab[chunk] * ATT_PAGE;
+    const int row0 = (chunk == c0 + 1 ? page1 : ptab[chunk]) * ATT_PAGE;
     uint8_t* kb = kvbuf + buf * C::BUF_BYTES;
     mbar_arrive_expect_tx(&bars[buf], C::BUF_BYTES);
     const uint64_t pol = policy_evict_last();
@@ -128,7 +113,44 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
       tma_load_2d(kb + C::KV_BYTES + b * (ATT_PAGE * BOXW * 2), mv, &bars[buf], h * HD + b * BOXW, row0, pol);
     }
   };
-  if (tid == 0 && c0 < c1) issue(c0, 0);
+  if (tid == 0) {
+    const int mv_ = max(max(s_info[2], s_info[3]), max(s_info[4], s_info[5]));
+    const int nch = (mv_ + ATT_PAGE - 1) / ATT_PAGE;
+    c1 = nch;
+    if (a.chunks_per_split > 0) {
+      c0 = min(nch, split * a.chunks_per_split);
+      c1 = min(nch, c0 + a.chunks_per_split);
+    }
+    s_info[0] = c0;
+    s_info[1] = c1;
+    // the first K / V chunk does not depend on Q: start its copy now
+    if (c0 < c1) {
+      if (c0 + 1 < c1) page1 = ptab[c0 + 1];
+      issue(c0, 0);
+    }
+  }
+  // Q tile -> shared memory (rows >= nq are zero); all of a thread's loads are issued first
+  {
+    constexpr int NQL = ATT_QTILE * (HD / 8) / 128;
+    uint4 v[NQL];
+#pragma unroll
+    for (int k = 0; k < NQL; ++k) {
+      const int i = tid + 128 * k;
+      const int r = i / (HD / 8), c = i % (HD / 8);
+      v[k] = r < nq ? __ldcg(reinterpret_cast<const uint4*>(a.q + (size_t)(t0 + r) * d + h * HD + c * 8))
+                    : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int k = 0; k < NQL; ++k) {
+      const int i = tid + 128 * k;
+      const int r = i / (HD / 8), c = i % (HD / 8);
+      *reinterpret_cast<uint4*>(qs + r * C::QSTRIDE + c * 8) = v[k];
+    }
+  }
+  named_bar_sync(bar_id, 128);
+  ATT_TR(1);
+  c0 = s_info[0];
+  c1 = s_info[1];
 
   // Q fragments (A operand) for this warp's 16 rows
   uint32_t qf[NKS][4];
@@ -157,6 +179,7 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
     if (tid == 0 && chunk + 1 < c1) issue(chunk + 1, buf ^ 1);
     const bool got = mbar_wait(&bars[buf], (uint32_t)(use[buf] & 1), a.err);
     __syncwarp();
+    if (chunk - c0 < 2) ATT_TR(2 + 2 * (chunk - c0));
     ++use[buf];
     if (!got) {
       ok = false;
@@ -211,7 +234,7 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
       o[j][2] *= alpha_b;
       o[j][3] *= alpha_b;
     }
-    uint32_t ph[4][4], pl[4][4];
+    uint32_t ph[4][4];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const float p0 = exp2f(s[j][0] - ua), p1 = exp2f(s[j][1] - ua);
@@ -219,10 +242,12 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
       l_a += p0 + p1;
       l_b += p2 + p3;
       const int kk = j >> 1, r = (j & 1) * 2;
-      split_f16(p0, p1, ph[kk][r], pl[kk][r]);
-      split_f16(p2, p3, ph[kk][r + 1], pl[kk][r + 1]);
+      const __half2 h01 = __floats2half2_rn(p0, p1), h23 = __floats2half2_rn(p2, p3);
+      ph[kk][r] = *reinterpret_cast<const uint32_t*>(&h01);
+      ph[kk][r + 1] = *reinterpret_cast<const uint32_t*>(&h23);
     }
-    // O += P V with P = hi + lo (fp16) and V fp16 (exactly the bf16-rounded values)
+    // O += P V with P in fp16 (11 significant bits; the row sum l uses the fp32 values) and V fp16
+    // (exactly the bf16-rounded values)
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk) {
 #pragma unroll
@@ -234,11 +259,10 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
         ldsm_x4_t(vbase + kv_off<HD>(key, ch), b0, b1, b2, b3);
         mma_f16_16816(o[2 * dd], ph[kk], b0, b1);
         mma_f16_16816(o[2 * dd + 1], ph[kk], b2, b3);
-        mma_f16_16816(o[2 * dd], pl[kk], b0, b1);
-        mma_f16_16816(o[2 * dd + 1], pl[kk], b2, b3);
       }
     }
     named_bar_sync(bar_id, 128);  // buffer `buf` may be refilled next iteration
+    if (chunk - c0 < 2) ATT_TR(3 + 2 * (chunk - c0));
   }
   if (!ok) {
     // the copy for the next chunk may still be in flight: wait for it (bounded) before returning
@@ -284,6 +308,8 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
         *reinterpret_cast<float2*>(a.part_ml + ((base + t0 + row_b) * a.n_heads + h) * 2) = make_float2(m_b, l_b);
     }
   }
+  ATT_TR(6);
+#undef ATT_TR
   return true;
 }
 

@@ -34,12 +34,12 @@ constexpr int ITEM_ROWS_FWD = 1024;   // item-code rows of the LM head (4 levels
 
 template <int BN>
 struct FCfg {
-  static constexpr int SA = BN == 128 ? 6 : 4;   // weight stages
-  static constexpr int SB = BN == 128 ? 5 : 3;   // activation stages
+  static constexpr int SA = BN == 128 ? 4 : 4;   // weight stages
+  static constexpr int SB = BN == 128 ? 3 : 3;   // activation stages
   static constexpr int A_BYTES = GEMM_BM * 128;
   static constexpr int B_BYTES = BN * 128;
   static constexpr int STAGING = 32 * GEMM_BM * 4;
-  static constexpr int MISC = 4096;
+  static constexpr int MISC = 8192;
   static constexpr int TMEM_COLS = 2 * BN;
 };
 
@@ -56,10 +56,12 @@ struct FLayout {
   static constexpr int EXTRA = (ATT_OFF + ATT_NEED > AFTER_STG) ? ((ATT_OFF + ATT_NEED - AFTER_STG + 1023) / 1024) * 1024 : 0;
   static constexpr int MISC_OFF = AFTER_STG + EXTRA;
   static constexpr int TOTAL = 1024 + MISC_OFF + C::MISC;
+  static_assert(C::SB * C::B_BYTES >= 8192 * 4, "a norm row (d <= 8192 floats) must fit in the activation ring");
 };
 
 struct GP {
   int epi;
+  bool to_dh;    // O / down projection: the product goes to dh (the next norm phase adds it to h)
   int M, K, m_tiles, n_tiles, kb, up_row0, rows;  // rows: valid tokens of the phase
   long long U;
   int Ge;        // CTAs that receive units: min(G, U) (the others idle in this phase)
@@ -73,6 +75,7 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
   g.layer = gi / 4;
   g.up_row0 = 0;
   g.rows = p.T;
+  g.to_dh = false;
   if (gi == 4 * L) {
     g.epi = EPI_F32;
     g.M = ITEM_ROWS_FWD;
@@ -89,7 +92,8 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
       g.K = p.d;
       g.mapB = act0;
     } else if (k == 1) {
-      g.epi = EPI_RESID;
+      g.epi = EPI_F32;
+      g.to_dh = true;
       g.M = p.d;
       g.K = p.d;
       g.mapB = act0 + 1;
@@ -100,7 +104,8 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
       g.up_row0 = p.ffn;
       g.mapB = act0;
     } else {
-      g.epi = EPI_RESID;
+      g.epi = EPI_F32;
+      g.to_dh = true;
       g.M = p.d;
       g.K = p.ffn;
       g.mapB = act0 + 2;
@@ -161,6 +166,31 @@ __device__ bool grid_wait(const FwdParams& p, int k) {
   }
 }
 
+__device__ __forceinline__ void st_release_cta(int* a, int v) {
+  asm volatile("st.release.cta.shared.u32 [%0], %1;" ::"r"(smem_u32(a)), "r"(v) : "memory");
+}
+__device__ __forceinline__ int ld_acquire_cta(const int* a) {
+  int v;
+  asm volatile("ld.acquire.cta.shared.u32 %0, [%1];" : "=r"(v) : "r"(smem_u32(a)) : "memory");
+  return v;
+}
+// Waits until the shared counter reaches `target` (bounded; false on timeout or a raised error).
+__device__ bool cta_count_wait(const int* cnt, int target, unsigned* err) {
+  if (ld_acquire_cta(cnt) >= target) return true;
+  const unsigned long long t0 = globaltimer_ns();
+  for (unsigned it = 1;; ++it) {
+    __nanosleep(32);
+    if (ld_acquire_cta(cnt) >= target) return true;
+    if ((it & 1023u) == 0u) {
+      if (err_set(err)) return false;
+      if (globaltimer_ns() - t0 > kWaitBudgetNs) {
+        set_error(err, ATSPEED_DEV_ERR_TIMEOUT);
+        return false;
+      }
+    }
+  }
+}
+
 // mbarrier wait that also gives up as soon as an error is raised anywhere
 __device__ bool mwait(uint64_t* bar, uint32_t parity, unsigned* err) {
   if (mbar_try_wait(bar, parity)) return true;
@@ -177,18 +207,14 @@ __device__ bool mwait(uint64_t* bar, uint32_t parity, unsigned* err) {
   }
 }
 
-template <int BN, int EPI>
-__device__ __forceinline__ void epi_dispatch_t(const GemmArgs& a, const float* st, int mt, int nt, int ch, int t) {
-  epi_chunk<BN, EPI>(a, st, mt, nt, ch, t);
-}
 template <int BN>
-__device__ __forceinline__ void epi_dispatch(int epi, const GemmArgs& a, const float* st, int mt, int nt, int ch,
-                                             int t) {
+__device__ __noinline__ void epi_dispatch(int epi, const GemmArgs& a, const float* st, int mt, int nt, int ch,
+                                             int t, const int* tpos, const int* tkvr) {
   switch (epi) {
-    case EPI_F32: epi_dispatch_t<BN, EPI_F32>(a, st, mt, nt, ch, t); break;
-    case EPI_RESID: epi_dispatch_t<BN, EPI_RESID>(a, st, mt, nt, ch, t); break;
-    case EPI_SWIGLU: epi_dispatch_t<BN, EPI_SWIGLU>(a, st, mt, nt, ch, t); break;
-    default: epi_dispatch_t<BN, EPI_QKV>(a, st, mt, nt, ch, t); break;
+    case EPI_F32: epi_chunk<BN, EPI_F32>(a, st, mt, nt, ch, t, tpos, tkvr); break;
+    case EPI_RESID: epi_chunk<BN, EPI_RESID>(a, st, mt, nt, ch, t, tpos, tkvr); break;
+    case EPI_SWIGLU: epi_chunk<BN, EPI_SWIGLU>(a, st, mt, nt, ch, t, tpos, tkvr); break;
+    default: epi_chunk<BN, EPI_QKV>(a, st, mt, nt, ch, t, tpos, tkvr); break;
   }
 }
 
@@ -207,12 +233,12 @@ __device__ GemmArgs epi_args(const FwdParams& p, const GP& g) {
   a.q_out = p.q;
   a.k_cache = p.kc + p.layer_elems * g.layer;
   a.v_cache = p.vc + p.layer_elems * g.layer;
-  if (g.epi == EPI_F32) {
+  if (g.to_dh) {
+    a.out_f32 = p.dh;
+    a.ldo = p.d;
+  } else if (g.epi == EPI_F32) {
     a.out_f32 = p.logits;
     a.ldo = ITEM_ROWS_FWD;
-  } else if (g.epi == EPI_RESID) {
-    a.out_f32 = p.h;
-    a.ldo = p.d;
   } else if (g.epi == EPI_SWIGLU) {
     a.out_bf16 = p.act;
     a.ldo = p.ffn;
@@ -220,73 +246,372 @@ __device__ GemmArgs epi_args(const FwdParams& p, const GP& g) {
   return a;
 }
 
-// RMSNorm of rows (128 compute threads, two virtual threads each; the sums are the same, bit for
-// bit, as the 256-thread kernels'): mode 0 = embedding gather + norm (layer 0), 1 = norm of h,
-// 2 = final norm of the selected rows.  A row stays in registers between the two passes.
-constexpr int NORM_MAXC = 8;   // float4 chunks per virtual thread: d <= 8192
+// Parts of the tiles of n-tile nt in the O / down projection gi: toff[mt] .. toff[mt + 1] index
+// tslot, the workspace slots of m-tile mt's parts in k order; a whole tile (one part) has none: its
+// product is in dh.  At most G + d / 128 entries.
+constexpr int PART_TABLE_CAP = 512;
 
-__device__ void norm_phase(const FwdParams& p, int mode, const __nv_bfloat16* g, float* red, int ctid) {
+template <int BN>
+__device__ void build_part_table(const FwdParams& p, int gi, int nt, int* toff, int* tslot, int ctid) {
+  const GP g = gemm_phase(p, gi, BN);
+  named_bar_sync(1, 128);   // earlier readers of the table are done
+  int cnt = 0, c_first = 0;
+  long long tu0 = 0;
+  if (ctid < g.m_tiles) {
+    tu0 = (long long)(ctid * g.n_tiles + nt) * g.kb;
+    c_first = uowner(tu0, g.U, g.Ge);
+    cnt = uowner(tu0 + g.kb - 1, g.U, g.Ge) - c_first + 1;
+    if (cnt == 1) cnt = 0;
+    toff[ctid + 1] = cnt;
+  }
+  named_bar_sync(1, 128);
+  if (ctid == 0) {
+    toff[0] = 0;
+    for (int t = 1; t <= g.m_tiles; ++t) toff[t] += toff[t - 1];
+  }
+  named_bar_sync(1, 128);
+  if (ctid < g.m_tiles) {
+    for (int pi = 0; pi < cnt; ++pi) {
+      const int cc = c_first + pi;
+      const int e = toff[ctid] + pi;
+      if (e < PART_TABLE_CAP) tslot[e] = cc * 2 + (ustart(cc, g.U, g.Ge) >= tu0 ? 0 : 1);
+    }
+  }
+  if (ctid == 0 && toff[g.m_tiles] > PART_TABLE_CAP) set_error(p.err, ATSPEED_DEV_ERR_BOUNDS);
+  named_bar_sync(1, 128);
+}
+
+// RMSNorm of rows (128 compute threads).  mode 0 = embedding gather + norm (layer 0); 1 = residual
+// add h += (product of the preceding O / down projection gi_prev, summed from its parts in k order
+// starting from zero), then norm of h; 2 = the same for the selected rows only (final norm).  The
+// sum of squares runs over two virtual threads per thread in the order of the 256-thread kernels,
+// so the result is the same, bit for bit.  Between the passes the row is kept in shared memory
+// (`rowbuf`, d floats: the activation ring, idle during a norm phase).
+constexpr int NORM_NB = 4;   // float4 chunks per virtual thread in flight
+
+template <int BN>
+__device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const __nv_bfloat16* g, float* red,
+                                        float4* rowbuf, int ctid, int gi_prev, int* toff, int* tslot, int& tab_nt,
+                                        int ph) {
   const int rows = mode == 2 ? p.n_out : p.T;
   const int d = p.d, nc = d / 4;
-  const int w = ctid >> 5;
+  const int w = ctid >> 5, lane = ctid & 31;
   for (int r = blockIdx.x; r < rows; r += p.G) {
     const int src = mode == 2 ? p.out_rows[r] : r;
     float* hr = p.h + (size_t)src * d;
-    float4 v[2][NORM_MAXC];
     float ss[2] = {0.f, 0.f};
+    if (mode == 0) {
+      const __nv_bfloat16* er = p.embed + (size_t)p.tok[r] * d;
+      for (int k0 = 0; k0 * 256 < nc; k0 += NORM_NB) {
+        float4 v[2][NORM_NB];
 #pragma unroll
-    for (int s = 0; s < 2; ++s) {
+        for (int s = 0; s < 2; ++s) {
 #pragma unroll
-      for (int k = 0; k < NORM_MAXC; ++k) {
-        const int c = ctid + 128 * s + 256 * k;
-        if (c < nc) {
-          if (mode == 0) {
-            const uint2 raw = *reinterpret_cast<const uint2*>(p.embed + (size_t)p.tok[r] * d + 4 * c);
-            const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&raw);
-            const float2 f0 = __bfloat1622float2(b[0]), f1 = __bfloat1622float2(b[1]);
-            v[s][k] = make_float4(f0.x, f0.y, f1.x, f1.y);
-            *reinterpret_cast<float4*>(hr + 4 * c) = v[s][k];
-          } else {
-            v[s][k] = __ldcg(reinterpret_cast<const float4*>(hr) + c);
+          for (int k = 0; k < NORM_NB; ++k) {
+            const int c = ctid + 128 * s + 256 * (k0 + k);
+            if (c < nc) {
+              const uint2 raw = *reinterpret_cast<const uint2*>(er + 4 * c);
+              const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&raw);
+              const float2 f0 = __bfloat1622float2(b[0]), f1 = __bfloat1622float2(b[1]);
+              v[s][k] = make_float4(f0.x, f0.y, f1.x, f1.y);
+            }
+          }
+        }
+#pragma unroll
+        for (int s = 0; s < 2; ++s) {
+#pragma unroll
+          for (int k = 0; k < NORM_NB; ++k) {
+            const int c = ctid + 128 * s + 256 * (k0 + k);
+            if (c < nc) {
+              *reinterpret_cast<float4*>(hr + 4 * c) = v[s][k];
+              rowbuf[c] = v[s][k];
+              ss[s] += v[s][k].x * v[s][k].x;
+              ss[s] += v[s][k].y * v[s][k].y;
+              ss[s] += v[s][k].z * v[s][k].z;
+              ss[s] += v[s][k].w * v[s][k].w;
+            }
           }
         }
       }
+    } else {
+      const int nt = src / BN, j = src - nt * BN;
+      if (gi_prev * 65536 + nt != tab_nt) {
+        build_part_table<BN>(p, gi_prev, nt, toff, tslot, ctid);
+        tab_nt = gi_prev * 65536 + nt;
+      }
+      // h += product: warp w takes m-tiles w, w + 4, ...; a lane four rows of each
+      const int mtn = (d + GEMM_BM - 1) / GEMM_BM;
+      const float4* ws4 = reinterpret_cast<const float4*>(p.ws);
+      constexpr long long SLOT4 = GEMM_WS_SLOT_FLOATS / 4;
+      const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int t0 = w; t0 < mtn; t0 += 32) {
+        float4 acc[8], hv[8];
+        int P[8], o[8];
+        int Pm = 0;
 #pragma unroll
-      for (int k = 0; k < NORM_MAXC; ++k) {
-        const int c = ctid + 128 * s + 256 * k;
-        if (c < nc) {
-          ss[s] += v[s][k].x * v[s][k].x;
-          ss[s] += v[s][k].y * v[s][k].y;
-          ss[s] += v[s][k].z * v[s][k].z;
-          ss[s] += v[s][k].w * v[s][k].w;
+        for (int b = 0; b < 8; ++b) {
+          const int mt = t0 + 4 * b;
+          const bool in = mt < mtn && mt * GEMM_BM + 4 * lane < d;
+          P[b] = in ? toff[mt + 1] - toff[mt] : 0;
+          o[b] = in ? toff[mt] : 0;
+          const size_t e = (size_t)src * d + mt * GEMM_BM + 4 * lane;
+          hv[b] = in ? __ldcg(reinterpret_cast<const float4*>(p.h + e)) : zero;
+          acc[b] = (in && P[b] == 0) ? __ldcg(reinterpret_cast<const float4*>(p.dh + e)) : zero;
+          Pm = max(Pm, P[b]);
+        }
+#pragma unroll 2
+        for (int e = 0; e < Pm; ++e) {
+          float4 v[8];
+#pragma unroll
+          for (int b = 0; b < 8; ++b)
+            if (e < P[b]) v[b] = __ldcg(ws4 + (long long)tslot[o[b] + e] * SLOT4 + j * (GEMM_BM / 4) + lane);
+#pragma unroll
+          for (int b = 0; b < 8; ++b) {
+            if (e < P[b]) {
+              acc[b].x += v[b].x;
+              acc[b].y += v[b].y;
+              acc[b].z += v[b].z;
+              acc[b].w += v[b].w;
+            }
+          }
+        }
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+          const int mt = t0 + 4 * b;
+          if (mt < mtn && mt * GEMM_BM + 4 * lane < d) {
+            const float4 v = make_float4(hv[b].x + acc[b].x, hv[b].y + acc[b].y, hv[b].z + acc[b].z,
+                                         hv[b].w + acc[b].w);
+            *reinterpret_cast<float4*>(hr + mt * GEMM_BM + 4 * lane) = v;   // the updated residual stream
+            rowbuf[mt * (GEMM_BM / 4) + lane] = v;
+          }
+        }
+      }
+      named_bar_sync(1, 128);
+      if (p.trace && ctid == 0 && r == (int)blockIdx.x) p.trace[((size_t)4 * (7 * p.L + 2) + ph) * p.G + blockIdx.x] = globaltimer_ns();
+#pragma unroll
+      for (int s = 0; s < 2; ++s) {
+        for (int k = 0;; ++k) {
+          const int c = ctid + 128 * s + 256 * k;
+          if (c >= nc) break;
+          const float4 v = rowbuf[c];
+          ss[s] += v.x * v.x;
+          ss[s] += v.y * v.y;
+          ss[s] += v.z * v.z;
+          ss[s] += v.w * v.w;
         }
       }
     }
     const float sa = warp_sum(ss[0]), sb = warp_sum(ss[1]);
-    if ((ctid & 31) == 0) {
+    if (lane == 0) {
       red[w] = sa;
       red[w + 4] = sb;
     }
     named_bar_sync(1, 128);
+    if (p.trace && ctid == 0 && r == (int)blockIdx.x) p.trace[((size_t)5 * (7 * p.L + 2) + ph) * p.G + blockIdx.x] = globaltimer_ns();
     const float rs = 1.0f / sqrtf(rms_total(red) / (float)d + p.eps);
-#pragma unroll
-    for (int s = 0; s < 2; ++s) {
-#pragma unroll
-      for (int k = 0; k < NORM_MAXC; ++k) {
-        const int c = ctid + 128 * s + 256 * k;
-        if (c < nc) {
-          const uint2 graw = *reinterpret_cast<const uint2*>(g + 4 * c);
-          const __nv_bfloat162* gb = reinterpret_cast<const __nv_bfloat162*>(&graw);
-          const float2 g0 = __bfloat1622float2(gb[0]), g1 = __bfloat1622float2(gb[1]);
-          __nv_bfloat162 o[2];
-          o[0] = __floats2bfloat162_rn(v[s][k].x * rs * g0.x, v[s][k].y * rs * g0.y);
-          o[1] = __floats2bfloat162_rn(v[s][k].z * rs * g1.x, v[s][k].w * rs * g1.y);
-          *reinterpret_cast<uint2*>(p.x + (size_t)r * d + 4 * c) = *reinterpret_cast<uint2*>(o);
-        }
-      }
+    __nv_bfloat16* xr = p.x + (size_t)r * d;
+#pragma unroll 4
+    for (int c = ctid; c < nc; c += 128) {
+      const float4 v = rowbuf[c];
+      const uint2 graw = *reinterpret_cast<const uint2*>(g + 4 * c);
+      const __nv_bfloat162* gb = reinterpret_cast<const __nv_bfloat162*>(&graw);
+      const float2 g0 = __bfloat1622float2(gb[0]), g1 = __bfloat1622float2(gb[1]);
+      __nv_bfloat162 o[2];
+      o[0] = __floats2bfloat162_rn(v.x * rs * g0.x, v.y * rs * g0.y);
+      o[1] = __floats2bfloat162_rn(v.z * rs * g1.x, v.w * rs * g1.y);
+      *reinterpret_cast<uint2*>(xr + 4 * c) = *reinterpret_cast<uint2*>(o);
     }
     named_bar_sync(1, 128);
   }
+}
+
+// Tree attention of layer l: this CTA's work items (query tile, head, prefix split); the last split
+// of a (tile, head) to finish merges the splits.
+template <int HD>
+__device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* att_smem, uint64_t* att_bars, int* s_info,
+                                        int (&use_att)[2], int* flag, int ctid) {
+  const int c = blockIdx.x, G = p.G, L = p.L;
+  AttnArgs a = p.att_args;
+  a.k_cache = p.kc + p.layer_elems * l;
+  a.v_cache = p.vc + p.layer_elems * l;
+  const CUtensorMap* mk = p.maps + 4 * L + 2 * l;
+  const CUtensorMap* mv = mk + 1;
+  const int H = p.H, S = a.max_splits;
+  const int NP = 7 * L + 2, ph = 7 * l + 2;
+  int nit = 0;
+  for (int item = c; item < p.att_items; item += G, ++nit) {
+    const int tile = item / (H * S), rem = item % (H * S);
+    const int h = rem / S, split = rem % S;
+    unsigned long long* tr = (p.trace && nit == 0) ? p.trace + ((size_t)8 * NP + ph) * G + c : nullptr;
+    if (!attn_item<HD>(a, mk, mv, tile, h, split, att_smem, att_bars, s_info, use_att, ctid, 1, tr, (size_t)NP * G))
+      return false;
+    if (p.trace && ctid == 0 && nit < 2) p.trace[((size_t)(4 + 2 * nit) * NP + ph) * G + c] = globaltimer_ns();
+    if (a.direct) continue;
+    const int S_u = a.user_splits[a.qt_user[tile]];
+    if (split >= S_u) continue;
+    __threadfence();
+    named_bar_sync(1, 128);
+    if (ctid == 0) {
+      const int old = atomicAdd(&p.att_counters[tile * H + h], 1);
+      const int last = old == S_u - 1;
+      if (last) {
+        p.att_counters[tile * H + h] = 0;
+        __threadfence();
+      }
+      *flag = last;
+    }
+    named_bar_sync(1, 128);
+    if (*flag) attn_combine_tile<HD>(a, tile, h, ctid);
+    named_bar_sync(1, 128);
+    if (p.trace && ctid == 0 && nit < 2) p.trace[((size_t)(5 + 2 * nit) * NP + ph) * G + c] = globaltimer_ns();
+  }
+  return true;
+}
+
+// GEMM phase gi (program phase ph), compute-warp side.  For each of this CTA's segments, wait for
+// its accumulator, then:
+//  * O / down projections (to_dh): a whole tile goes to dh, a split tile's part to this CTA's
+//    workspace slot ([token][row] layout); the next norm phase sums the parts (no reduction here);
+//  * other GEMMs: a whole tile runs the fused epilogue; for a split tile, if every other part is
+//    already published this CTA is the last one and sums the parts with its own part read straight
+//    from TMEM; otherwise it publishes its part and the last CTA to arrive does the sum.
+// Parts are always summed in k order starting from zero, whichever CTA sums them.  Kept out of
+// line so that the epilogue gets its own register allocation.
+template <int BN>
+__device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, float* staging, uint64_t* tfull,
+                                            uint64_t* tempty, int* flag, int* part_slot, int* tpos, int* tkvr,
+                                            uint32_t tmem_base, int ctid, int& si) {
+  const int c = blockIdx.x, G = p.G, NP = 7 * p.L + 2;
+  const int lane = ctid & 31, q = ctid >> 5, m = ctid;   // warp 4 + q reads TMEM lane quadrant q
+  const GP g = gemm_phase(p, gi, BN);
+  const GemmArgs ea = epi_args(p, g);
+  const int kb = g.kb;
+  long long u0, u1;
+  crange(g, c, u0, u1);
+  int seg = 0;
+  for (long long u = u0; u < u1; ++si, ++seg) {
+    const int tile = (int)(u / kb);
+    const int k0 = (int)(u % kb);
+    const long long len = (kb - k0) < (u1 - u) ? (kb - k0) : (u1 - u);
+    const int k1 = k0 + (int)len;
+    u += len;
+    const int acc = si & 1, use = si >> 1;
+    const int m_tile = tile / g.n_tiles, n_tile = tile % g.n_tiles;
+    const bool whole = (k0 == 0 && k1 == kb);
+    if (g.epi == EPI_QKV) load_tok_tables<BN>(ea, n_tile, tpos, tkvr, ctid);
+    long long tu0 = 0;
+    int c_first = 0, parts = 1;
+    if (!whole && !g.to_dh) {
+      tu0 = (long long)tile * kb;
+      c_first = uowner(tu0, g.U, g.Ge);
+      parts = uowner(tu0 + kb - 1, g.U, g.Ge) - c_first + 1;
+      for (int pi = ctid; pi < parts; pi += 128) {
+        const int cc = c_first + pi;
+        part_slot[pi] = cc * 2 + (ustart(cc, g.U, g.Ge) >= tu0 ? 0 : 1);
+      }
+    }
+    const bool got = mwait(&tfull[acc], (uint32_t)(use & 1), p.err);
+    __syncwarp();
+    if (!got) return false;
+    tc_fence_after();
+    if (p.trace && ctid == 0) p.trace[((size_t)4 * NP + ph) * G + c] = globaltimer_ns();
+    const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+    const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
+    const int row = m_tile * GEMM_BM + m;
+    if (g.to_dh) {
+      float* dst;
+      size_t ld;
+      if (whole) {
+        dst = p.dh + (size_t)n_tile * BN * p.d + row;
+        ld = (size_t)p.d;
+      } else {
+        dst = p.ws + ((long long)c * 2 + (seg == 0 ? 0 : 1)) * GEMM_WS_SLOT_FLOATS + m;
+        ld = GEMM_BM;
+      }
+      for (int ch = 0; ch < nch; ++ch) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tb + ch * 32, r);
+        tmem_ld_wait();
+        const int nv = min(32, g.rows - n_tile * BN - ch * 32);
+        if (!whole || row < g.M) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (j < nv) __stcg(dst + (size_t)(ch * 32 + j) * ld, __uint_as_float(r[j]));
+        }
+      }
+      tc_fence_before();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      continue;
+    }
+    if (whole) {
+      for (int ch = 0; ch < nch; ++ch) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tb + ch * 32, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = __uint_as_float(r[j]);
+        named_bar_sync(1, 128);
+        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid, tpos, tkvr);
+        named_bar_sync(1, 128);
+      }
+      tc_fence_before();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      continue;
+    }
+    // split tile: are the other parts all published already?
+    if (ctid == 0) *flag = (int)ld_acquire_u32(reinterpret_cast<const unsigned*>(&p.counters[tile])) == parts - 1;
+    named_bar_sync(1, 128);
+    if (*flag) {
+      // last part: nobody else touches this tile's counter in this phase
+      if (ctid == 0) p.counters[tile] = 0;
+      if (p.trace && ctid == 0) p.trace[((size_t)6 * NP + ph) * G + c] = globaltimer_ns();
+      const int own = c - c_first;
+      for (int ch = 0; ch < nch; ++ch) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tb + ch * 32, r);
+        tmem_ld_wait();
+        ws_reduce_chunk_own(p.ws, part_slot, parts, own, r, ch, m, staging);
+        named_bar_sync(1, 128);
+        if (p.trace && ctid == 0 && ch < 4) p.trace[((size_t)(8 + 2 * ch) * NP + ph) * G + c] = globaltimer_ns();
+        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid, tpos, tkvr);
+        named_bar_sync(1, 128);
+        if (p.trace && ctid == 0 && ch < 4) p.trace[((size_t)(9 + 2 * ch) * NP + ph) * G + c] = globaltimer_ns();
+      }
+      tc_fence_before();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      continue;
+    }
+    const long long slot = (long long)c * 2 + (seg == 0 ? 0 : 1);
+    ws_store_partial(p.ws + slot * GEMM_WS_SLOT_FLOATS, tb, nch, m);
+    tc_fence_before();
+    if (lane == 0) mbar_arrive(&tempty[acc]);
+    __threadfence();
+    named_bar_sync(1, 128);
+    if (p.trace && ctid == 0) p.trace[((size_t)5 * NP + ph) * G + c] = globaltimer_ns();
+    if (ctid == 0) {
+      const int old = atomicAdd(&p.counters[tile], 1);
+      const int last = (old == parts - 1);
+      if (last) {
+        p.counters[tile] = 0;
+        __threadfence();
+      }
+      *flag = last;
+    }
+    named_bar_sync(1, 128);
+    if (p.trace && ctid == 0) p.trace[((size_t)6 * NP + ph) * G + c] = globaltimer_ns();
+    if (*flag) {
+      for (int ch = 0; ch < nch; ++ch) {
+        ws_reduce_chunk(p.ws, part_slot, parts, ch, m, staging);
+        named_bar_sync(1, 128);
+        if (p.trace && ctid == 0 && ch < 4) p.trace[((size_t)(8 + 2 * ch) * NP + ph) * G + c] = globaltimer_ns();
+        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid, tpos, tkvr);
+        named_bar_sync(1, 128);
+        if (p.trace && ctid == 0 && ch < 4) p.trace[((size_t)(9 + 2 * ch) * NP + ph) * G + c] = globaltimer_ns();
+      }
+    }
+    named_bar_sync(1, 128);  // flag and part_slot are reused by the next segment
+  }
+  return true;
 }
 
 template <int HD, int BN>
@@ -299,6 +624,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
   uint8_t* ringB = smem + LY::B_OFF;
   float* staging = reinterpret_cast<float*>(smem + LY::STG_OFF);
   uint8_t* att_smem = smem + LY::ATT_OFF;
+  float4* rowbuf = reinterpret_cast<float4*>(ringB);   // norm phases: one row, d <= 8192 floats
   uint64_t* fullA = reinterpret_cast<uint64_t*>(smem + LY::MISC_OFF);
   uint64_t* emptyA = fullA + C::SA;
   uint64_t* fullB = emptyA + C::SA;
@@ -310,11 +636,19 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(att_bars + 2);
   int* flag = reinterpret_cast<int*>(tmem_slot + 1);
   int* failed = flag + 1;
-  int* lastA = failed + 1;                                        // [SA] parity of last fill, -1 none
+  int* go = failed + 1;   // count of GEMM phases whose input the compute warps have seen published
+  int* lastA = go + 1;                                            // [SA] parity of last fill, -1 none
   int* lastB = lastA + C::SA;                                     // [SB]
-  int* s_info = lastB + C::SB;                                    // 2 (attention)
-  float* red = reinterpret_cast<float*>(s_info + 2);              // 8
+  int* s_info = lastB + C::SB;                                    // 6 (attention)
+  float* red = reinterpret_cast<float*>(s_info + 6);              // 8
   int* part_slot = reinterpret_cast<int*>(red + 8);               // 256
+  int* tpos = part_slot + 256;                                    // [BN] QKV token tables
+  int* tkvr = tpos + 256;
+  int* toff = tkvr + 256;                                         // [65] part table (norm phases)
+  int* tslot = toff + 68;                                         // [PART_TABLE_CAP]
+  static_assert(8 * (2 * C::SA + 2 * C::SB + 7) + 4 * (4 + C::SA + C::SB + 6 + 8 + 256 + 512 + 68 + PART_TABLE_CAP) <=
+                    C::MISC,
+                "shared-memory misc area too small");
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x, G = p.G, L = p.L;
@@ -338,6 +672,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
       mbar_init(&att_bars[i], 1);
     }
     mbar_init(mma_done, 1);
+    *go = 0;
     *failed = 0;
     fence_mbar_init();
   }
@@ -397,11 +732,13 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
         const GP g = gemm_phase(p, gi, BN);
         long long u0, u1;
         crange(g, c, u0, u1);
-        if (u1 <= u0) continue;
-        if (!grid_wait(p, gemm_phase_index(gi, L) - 1)) {
+        // the compute warps pass the grid barrier that publishes this phase's input and count it in
+        // `go` (one grid poller per CTA)
+        if (!cta_count_wait(go, gi + 1, p.err)) {
           ok = false;
           break;
         }
+        if (u1 <= u0) continue;
         if (p.trace) p.trace[((size_t)1 * (7 * L + 2) + gi) * G + c] = globaltimer_ns();
         fence_proxy_async();
         const CUtensorMap* mB = p.maps + g.mapB;
@@ -483,6 +820,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
     const int m = q * 32 + lane;
     int si = 0;
     int use_att[2] = {0, 0};
+    int tab_nt = -1;   // (GEMM phase, n-tile) whose part table is in toff / tslot
     bool ok = true;
     for (int ph = 0; ph < NP && ok; ++ph) {
       // which phase is this?
@@ -507,11 +845,27 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
           kind = 4;
         }
       }
+      if ((kind == 3 || kind == 4) && ph > 0) {
+        // the part table of this CTA's first row does not depend on data: build it before the wait
+        const int r0 = blockIdx.x;
+        const bool fin = kind == 4 && l + 1 == L;
+        if (r0 < (fin ? p.n_out : p.T)) {
+          const int nt = (fin ? p.out_rows[r0] : r0) / BN;
+          const int gp = 4 * l + (kind == 3 ? 1 : 3);
+          if (gp * 65536 + nt != tab_nt) {
+            build_part_table<BN>(p, gp, nt, toff, tslot, ctid);
+            tab_nt = gp * 65536 + nt;
+          }
+        }
+      }
       if (ph > 0) {
         // Barrier ph-1 must be complete before this CTA can arrive at barrier ph: the arrival counter
         // is shared by all barriers, so an early arrival would count towards the previous one.
         // (Non-GEMM phases also read what the previous phase wrote.)
-        if (ctid == 0) *flag = grid_wait(p, ph - 1) ? 1 : 0;
+        if (ctid == 0) {
+          *flag = grid_wait(p, ph - 1) ? 1 : 0;
+          if (*flag && kind == 1) st_release_cta(go, gi + 1);
+        }
         named_bar_sync(1, 128);
         if (!*flag) {
           ok = false;
@@ -520,141 +874,21 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
         fence_proxy_async();
         named_bar_sync(1, 128);
       }
-      if (kind == 0) {
-        norm_phase(p, 0, p.attn_norm[0], red, ctid);
-      } else if (kind == 3) {
-        norm_phase(p, 1, p.mlp_norm[l], red, ctid);
-      } else if (kind == 4) {
-        if (l + 1 < L)
-          norm_phase(p, 1, p.attn_norm[l + 1], red, ctid);
-        else
-          norm_phase(p, 2, p.final_norm, red, ctid);
+      if (kind == 0 || kind == 3 || kind == 4) {
+        const int nmode = kind == 0 ? 0 : (kind == 4 && l + 1 == L) ? 2 : 1;
+        const __nv_bfloat16* ng = kind == 0 ? p.attn_norm[0] : kind == 3 ? p.mlp_norm[l]
+                                  : (l + 1 < L ? p.attn_norm[l + 1] : p.final_norm);
+        norm_phase<BN>(p, nmode, ng, red, rowbuf, ctid, 4 * l + (kind == 3 ? 1 : 3), toff, tslot, tab_nt, ph);
       } else if (kind == 2) {
-        AttnArgs a = p.att_args;
-        a.k_cache = p.kc + p.layer_elems * l;
-        a.v_cache = p.vc + p.layer_elems * l;
-        const CUtensorMap* mk = p.maps + 4 * L + 2 * l;
-        const CUtensorMap* mv = mk + 1;
-        const int H = p.H, S = a.max_splits;
-        for (int item = c; item < p.att_items && ok; item += G) {
-          const int tile = item / (H * S), rem = item % (H * S);
-          const int h = rem / S, split = rem % S;
-          if (!attn_item<HD>(a, mk, mv, tile, h, split, att_smem, att_bars, s_info, use_att, ctid, 1)) {
-            ok = false;
-            break;
-          }
-          if (a.direct) continue;
-          const int S_u = a.user_splits[a.qt_user[tile]];
-          if (split >= S_u) continue;
-          __threadfence();
-          named_bar_sync(1, 128);
-          if (ctid == 0) {
-            const int old = atomicAdd(&p.att_counters[tile * H + h], 1);
-            const int last = old == S_u - 1;
-            if (last) {
-              p.att_counters[tile * H + h] = 0;
-              __threadfence();
-            }
-            *flag = last;
-          }
-          named_bar_sync(1, 128);
-          if (*flag) attn_combine_tile<HD>(a, tile, h, ctid);
-          named_bar_sync(1, 128);
+        if (!attn_phase<HD>(p, l, att_smem, att_bars, s_info, use_att, flag, ctid)) {
+          ok = false;
+          break;
         }
       } else {
-        // ---- GEMM epilogue for this CTA's segments of phase gi
-        const GP g = gemm_phase(p, gi, BN);
-        const GemmArgs ea = epi_args(p, g);
-        const int kb = g.kb;
-        long long u0, u1;
-        crange(g, c, u0, u1);
-        int seg = 0;
-        for (long long u = u0; u < u1 && ok; ++si, ++seg) {
-          const int tile = (int)(u / kb);
-          const int k0 = (int)(u % kb);
-          const long long len = (kb - k0) < (u1 - u) ? (kb - k0) : (u1 - u);
-          const int k1 = k0 + (int)len;
-          u += len;
-          const int acc = si & 1, use = si >> 1;
-          const bool got = mwait(&tfull[acc], (uint32_t)(use & 1), p.err);
-          __syncwarp();
-          if (!got) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const int m_tile = tile / g.n_tiles, n_tile = tile % g.n_tiles;
-          const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-          const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
-          if (k0 == 0 && k1 == kb) {
-            for (int ch = 0; ch < nch; ++ch) {
-              uint32_t r[32];
-              tmem_ld_32x32b_x32(tb + ch * 32, r);
-              tmem_ld_wait();
-#pragma unroll
-              for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = __uint_as_float(r[j]);
-              named_bar_sync(1, 128);
-              epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid);
-              named_bar_sync(1, 128);
-            }
-            tc_fence_before();
-            if (lane == 0) mbar_arrive(&tempty[acc]);
-          } else {
-            const long long slot = (long long)c * 2 + (seg == 0 ? 0 : 1);
-            float* wsl = p.ws + slot * GEMM_WS_SLOT_FLOATS;
-            for (int ch = 0; ch < nch; ++ch) {
-              uint32_t r[32];
-              tmem_ld_32x32b_x32(tb + ch * 32, r);
-              tmem_ld_wait();
-#pragma unroll
-              for (int j = 0; j < 32; ++j) __stcg(&wsl[(ch * 32 + j) * GEMM_BM + m], __uint_as_float(r[j]));
-            }
-            tc_fence_before();
-            if (lane == 0) mbar_arrive(&tempty[acc]);
-            __threadfence();
-            named_bar_sync(1, 128);
-            const long long tu0 = (long long)tile * kb;
-            const int c_first = uowner(tu0, g.U, g.Ge);
-            const int c_last = uowner(tu0 + kb - 1, g.U, g.Ge);
-            const int parts = c_last - c_first + 1;
-            if (ctid == 0) {
-              const int old = atomicAdd(&p.counters[tile], 1);
-              const int last = (old == parts - 1);
-              if (last) {
-                p.counters[tile] = 0;
-                __threadfence();
-              }
-              *flag = last;
-            }
-            for (int pi = ctid; pi < parts; pi += 128) {
-              const int cc = c_first + pi;
-              part_slot[pi] = cc * 2 + (ustart(cc, g.U, g.Ge) >= tu0 ? 0 : 1);
-            }
-            named_bar_sync(1, 128);
-            if (*flag) {
-              for (int ch = 0; ch < nch; ++ch) {
-                float accv[32];
-#pragma unroll
-                for (int j = 0; j < 32; ++j) accv[j] = 0.f;
-                for (int pi = 0; pi < parts; ++pi) {
-                  const float* src = p.ws + (long long)part_slot[pi] * GEMM_WS_SLOT_FLOATS + (ch * 32) * GEMM_BM + m;
-                  float v[32];
-#pragma unroll
-                  for (int j = 0; j < 32; ++j) v[j] = __ldcg(src + j * GEMM_BM);
-#pragma unroll
-                  for (int j = 0; j < 32; ++j) accv[j] += v[j];
-                }
-#pragma unroll
-                for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = accv[j];
-                named_bar_sync(1, 128);
-                epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid);
-                named_bar_sync(1, 128);
-              }
-            }
-            named_bar_sync(1, 128);  // flag and part_slot are reused by the next segment
-          }
+        if (!gemm_epi_phase<BN>(p, gi, ph, staging, tfull, tempty, flag, part_slot, tpos, tkvr, tmem_base, ctid, si)) {
+          ok = false;
+          break;
         }
-        if (!ok) break;
       }
       if (p.trace && ctid == 0) p.trace[(size_t)ph * G + c] = globaltimer_ns();
       // publish this phase: this CTA's generic-proxy stores must be visible to the other CTAs'

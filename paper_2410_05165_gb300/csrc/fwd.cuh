@@ -34,6 +34,7 @@ struct FwdParams {
   const __nv_bfloat16* embed;
   // activations
   float* h;                 // [T][d] fp32 residual stream
+  float* dh;                // [T][d] fp32 product of the last O / down projection, added to h by the norm
   __nv_bfloat16* x;         // [Xrows][d] normalised rows (GEMM B operand)
   __nv_bfloat16* q;         // [T][d]
   __nv_bfloat16* att;       // [Xrows][d]
@@ -60,7 +61,7 @@ struct FwdParams {
   // grid barrier: monotonic arrival counter, zeroed before the launch
   unsigned int* bar;
   unsigned int* err;
-  unsigned long long* trace;  // optional [phases][G] globaltimer at the end of each phase, or null
+  unsigned long long* trace;  // optional [16][phases][G] globaltimer stamps (phase end, producer and epilogue milestones), or null
 };
 
 // Shared memory the persistent kernel needs for (head_dim, token tile) = (hd, bn).

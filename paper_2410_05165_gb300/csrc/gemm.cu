@@ -36,7 +36,7 @@ struct Cfg {
   static constexpr int B_BYTES = BN * 128;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGING_FLOATS = 32 * BM;
-  static constexpr int BAR_BYTES = 256 + 1024;  // barriers, flags, split-part slot table
+  static constexpr int BAR_BYTES = 256 + 1024 + 2048;  // barriers, flags, split-part slot table, token tables
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_FLOATS * 4 + BAR_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
 };
@@ -75,6 +75,8 @@ __global__ void __launch_bounds__(192, 1)
   int* failed = flag + 1;
   int* last_fill = failed + 1;  // [STAGES]: parity of the last fill issued per stage, -1 if none
   int* part_slot = last_fill + 8;  // [<= 256] workspace slots of a split tile's parts
+  int* tpos = part_slot + 256;     // [BN] QKV epilogue token tables of the current n-tile
+  int* tkvr = tpos + 256;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x;
@@ -233,6 +235,7 @@ __global__ void __launch_bounds__(192, 1)
       }
       tc_fence_after();
       const int m_tile = tile / p.n_tiles, n_tile = tile % p.n_tiles;
+      if constexpr (EPI == EPI_QKV) load_tok_tables<BN>(p.a, n_tile, tpos, tkvr, ep_tid);
       const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       // 32-token chunks that hold at least one valid token (the rest are padding)
       const int nch = min(BN / 32, (p.a.T - n_tile * BN + 31) / 32);
@@ -244,21 +247,14 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
           for (int j = 0; j < 32; ++j) staging[j * BM + m] = __uint_as_float(r[j]);
           named_bar_sync(1, 128);
-          epi_chunk<BN, EPI>(p.a, staging, m_tile, n_tile, ch, ep_tid);
+          epi_chunk<BN, EPI>(p.a, staging, m_tile, n_tile, ch, ep_tid, tpos, tkvr);
           named_bar_sync(1, 128);
         }
         tc_fence_before();
         if (lane == 0) mbar_arrive(&tempty[acc]);
       } else {
         const long long slot = (long long)c * 2 + (si == 0 ? 0 : 1);
-        float* wsl = p.ws + slot * WS_SLOT_FLOATS;
-        for (int ch = 0; ch < nch; ++ch) {
-          uint32_t r[32];
-          tmem_ld_32x32b_x32(tb + ch * 32, r);
-          tmem_ld_wait();
-#pragma unroll
-          for (int j = 0; j < 32; ++j) __stcg(&wsl[(ch * 32 + j) * BM + m], __uint_as_float(r[j]));
-        }
+        ws_store_partial(p.ws + slot * WS_SLOT_FLOATS, tb, nch, m);
         tc_fence_before();
         if (lane == 0) mbar_arrive(&tempty[acc]);
         __threadfence();
@@ -284,21 +280,9 @@ __global__ void __launch_bounds__(192, 1)
         named_bar_sync(1, 128);
         if (*flag) {
           for (int ch = 0; ch < nch; ++ch) {
-            float accv[32];
-#pragma unroll
-            for (int j = 0; j < 32; ++j) accv[j] = 0.f;
-            for (int pi = 0; pi < parts; ++pi) {
-              const float* src = p.ws + (long long)part_slot[pi] * WS_SLOT_FLOATS + (ch * 32) * BM + m;
-              float v[32];
-#pragma unroll
-              for (int j = 0; j < 32; ++j) v[j] = __ldcg(src + j * BM);   // 32 independent loads in flight
-#pragma unroll
-              for (int j = 0; j < 32; ++j) accv[j] += v[j];
-            }
-#pragma unroll
-            for (int j = 0; j < 32; ++j) staging[j * BM + m] = accv[j];
+            ws_reduce_chunk(p.ws, part_slot, parts, ch, m, staging);
             named_bar_sync(1, 128);
-            epi_chunk<BN, EPI>(p.a, staging, m_tile, n_tile, ch, ep_tid);
+            epi_chunk<BN, EPI>(p.a, staging, m_tile, n_tile, ch, ep_tid, tpos, tkvr);
             named_bar_sync(1, 128);
           }
         }

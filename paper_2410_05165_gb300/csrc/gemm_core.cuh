@@ -9,12 +9,71 @@ constexpr int GEMM_BK = 64;    // bf16 elements per 128-byte swizzle row (one k-
 constexpr int GEMM_BM = 128;   // weight rows per tile (MMA M)
 constexpr int GEMM_WS_SLOT_FLOATS = 256 * 128;
 
+// Per-token data of the QKV epilogue for the BN tokens of n-tile n_tile (rotary position and cache
+// row), copied to shared memory when a segment starts so that the epilogue's loads do not wait on
+// them.  Callers synchronise the 128 threads before the first chunk's epilogue.
+template <int BN>
+__device__ __forceinline__ void load_tok_tables(const GemmArgs& a, int n_tile, int* tpos, int* tkvr, int ep_tid) {
+  for (int j = ep_tid; j < BN; j += 128) {
+    const int tok = n_tile * BN + j;
+    tpos[j] = tok < a.T ? a.pos[tok] : 0;
+    tkvr[j] = tok < a.T ? a.kv_row[tok] : 0;
+  }
+}
+
 // st: staging [32 tokens][128 rows] fp32 of one chunk; 128 threads (ep_tid) write the outputs.
+// tpos / tkvr: the n-tile's token tables (EPI_QKV only).
 template <int BN, int EPI>
 __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, int m_tile, int n_tile, int ch,
-                                          int ep_tid) {
+                                          int ep_tid, const int* tpos, const int* tkvr) {
   const int tok0 = n_tile * BN + ch * 32;
-  if constexpr (EPI == EPI_SWIGLU) {
+  if constexpr (EPI == EPI_QKV) {
+    // rows of q | k | v.  Thread = (rotation pair, token parity): pair (i, i + hd/2) of one head
+    // shares its cos / sin, and the thread rotates both rows (rotate-half RoPE) for tokens
+    // (ep_tid >> 6) + 2k; k / v rows go to their cache rows, v rounded to bf16 and kept as fp16.
+    const int d = a.d_model, hd = a.head_dim, half = hd >> 1;
+    const int pi = ep_tid & 63, n0 = ep_tid >> 6;
+    const int hh = pi / half, i = pi - hh * half;
+    const int r_lo = hh * hd + i, r_hi = r_lo + half;     // rows within the tile
+    const int row = m_tile * GEMM_BM + r_lo;
+    if (row >= a.M) return;                                // padding rows of the last tile
+    const int region = row / d;
+    const int f_lo = row - region * d, f_hi = f_lo + half;
+    const int nv = min(32, a.T - tok0);
+    const int tt0 = ch * 32;                               // token-table index of the chunk's first token
+    if (region == 2) {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const int n = n0 + 2 * k;
+        if (n < nv) {
+          __half* vr = a.v_cache + (size_t)tkvr[tt0 + n] * d;
+          vr[f_lo] = __float2half_rn(bf16_round(st[n * GEMM_BM + r_lo]));
+          vr[f_hi] = __float2half_rn(bf16_round(st[n * GEMM_BM + r_hi]));
+        }
+      }
+    } else {
+      float cth[16], sth[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const int n = n0 + 2 * k;
+        const size_t cs = (size_t)tpos[tt0 + (n < nv ? n : 0)] * half + i;
+        cth[k] = a.rope_cos[cs];
+        sth[k] = a.rope_sin[cs];
+      }
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const int n = n0 + 2 * k;
+        if (n < nv) {
+          const float x_lo = st[n * GEMM_BM + r_lo], x_hi = st[n * GEMM_BM + r_hi];
+          const __nv_bfloat16 o_lo = __float2bfloat16_rn(x_lo * cth[k] - x_hi * sth[k]);
+          const __nv_bfloat16 o_hi = __float2bfloat16_rn(x_hi * cth[k] + x_lo * sth[k]);
+          __nv_bfloat16* orow = region == 0 ? a.q_out + (size_t)(tok0 + n) * d : a.k_cache + (size_t)tkvr[tt0 + n] * d;
+          orow[f_lo] = o_lo;
+          orow[f_hi] = o_hi;
+        }
+      }
+    }
+  } else if constexpr (EPI == EPI_SWIGLU) {
     // thread owns feature i of the tile and tokens (ep_tid >> 6) + 2k
     const int i = ep_tid & 63, n0 = ep_tid >> 6;
     __nv_bfloat16* out = a.out_bf16 + m_tile * 64 + i;
@@ -49,34 +108,102 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, in
 #pragma unroll
       for (int n = 0; n < 32; ++n)
         if (n < nv) base[(size_t)n * a.ldo] = old[n] + st[n * GEMM_BM + m];
-    } else {  // EPI_QKV: rows of q | k | v; RoPE (rotate-half) on q and k, k / v to their cache rows
-      const int d = a.d_model, hd = a.head_dim, half = hd >> 1;
-      const int region = row / d;
-      const int f = row - region * d;
-      const int i = f & (hd - 1);
-      const bool lo = i < half;
-      const int ii = lo ? i : i - half;
-      const int partner = lo ? m + half : m - half;
-#pragma unroll 4
-      for (int n = 0; n < nv; ++n) {
-        const int tok = tok0 + n;
-        const float v = st[n * GEMM_BM + m];
-        if (region == 2) {
-          a.v_cache[(size_t)a.kv_row[tok] * d + f] = __float2half_rn(bf16_round(v));
-          continue;
+    }
+  }
+}
+
+// ---- split-K partials (stream-K tiles shared by several CTAs)
+// A workspace slot holds one CTA's fp32 partial of a 128-row tile for up to 256 tokens, laid out
+// [token/4][row][4] so that a thread (one weight row) moves four tokens per 16-byte access.
+
+// TMEM accumulator (this thread's lane = row m) -> workspace slot, chunks [0, nch)
+__device__ __forceinline__ void ws_store_partial(float* wsl, uint32_t tb, int nch, int m) {
+  float4* w4 = reinterpret_cast<float4*>(wsl);
+  for (int ch = 0; ch < nch; ++ch) {
+    uint32_t r[32];
+    tmem_ld_32x32b_x32(tb + ch * 32, r);
+    tmem_ld_wait();
+#pragma unroll
+    for (int j4 = 0; j4 < 8; ++j4)
+      __stcg(&w4[(ch * 8 + j4) * GEMM_BM + m],
+             make_float4(__uint_as_float(r[4 * j4]), __uint_as_float(r[4 * j4 + 1]), __uint_as_float(r[4 * j4 + 2]),
+                         __uint_as_float(r[4 * j4 + 3])));
+  }
+}
+
+// Sum, in k order (part 0 first, starting from zero), of chunk ch of the parts in `slot` -> this
+// thread's row m of the staging buffer [32 tokens][128 rows].  Up to four parts are in flight at once.
+__device__ __forceinline__ void ws_reduce_chunk(const float* ws, const int* slot, int parts, int ch, int m,
+                                                float* staging) {
+  float acc[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) acc[j] = 0.f;
+  const float4* w4 = reinterpret_cast<const float4*>(ws);
+  constexpr long long SLOT4 = GEMM_WS_SLOT_FLOATS / 4;
+  for (int p0 = 0; p0 < parts; p0 += 4) {
+    float4 v[4][8];
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      if (p0 + b < parts) {
+        const float4* src = w4 + (long long)slot[p0 + b] * SLOT4 + (ch * 8) * GEMM_BM + m;
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) v[b][j4] = __ldcg(src + j4 * GEMM_BM);
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      if (p0 + b < parts) {
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) {
+          acc[4 * j4] += v[b][j4].x;
+          acc[4 * j4 + 1] += v[b][j4].y;
+          acc[4 * j4 + 2] += v[b][j4].z;
+          acc[4 * j4 + 3] += v[b][j4].w;
         }
-        const size_t cs = (size_t)a.pos[tok] * half + ii;
-        const float cth = a.rope_cos[cs], sth = a.rope_sin[cs];
-        const float x2 = st[n * GEMM_BM + partner];
-        const float out = lo ? v * cth - x2 * sth : v * cth + x2 * sth;
-        const __nv_bfloat16 ob = __float2bfloat16_rn(out);
-        if (region == 0)
-          a.q_out[(size_t)tok * d + f] = ob;
-        else
-          a.k_cache[(size_t)a.kv_row[tok] * d + f] = ob;
       }
     }
   }
+#pragma unroll
+  for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = acc[j];
+}
+
+// As ws_reduce_chunk, with part `own` of the sum taken from registers (this CTA's accumulator, 32
+// tokens of row m) instead of the workspace.  Two parts are in flight at once.
+__device__ __forceinline__ void ws_reduce_chunk_own(const float* ws, const int* slot, int parts, int own,
+                                                    const uint32_t (&r)[32], int ch, int m, float* staging) {
+  float acc[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) acc[j] = 0.f;
+  const float4* w4 = reinterpret_cast<const float4*>(ws);
+  constexpr long long SLOT4 = GEMM_WS_SLOT_FLOATS / 4;
+  for (int p0 = 0; p0 < parts; p0 += 2) {
+    float4 v[2][8];
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      if (p0 + b < parts && p0 + b != own) {
+        const float4* src = w4 + (long long)slot[p0 + b] * SLOT4 + (ch * 8) * GEMM_BM + m;
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) v[b][j4] = __ldcg(src + j4 * GEMM_BM);
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      if (p0 + b == own) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) acc[j] += __uint_as_float(r[j]);
+      } else if (p0 + b < parts) {
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) {
+          acc[4 * j4] += v[b][j4].x;
+          acc[4 * j4 + 1] += v[b][j4].y;
+          acc[4 * j4 + 2] += v[b][j4].z;
+          acc[4 * j4 + 3] += v[b][j4].w;
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = acc[j];
 }
 
 }  // namespace atspeed
