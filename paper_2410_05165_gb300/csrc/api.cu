@@ -135,7 +135,7 @@ struct atspeed_ctx {
   std::vector<ProfRec> prof_recs;
   std::vector<cudaEvent_t> prof_pool;
   long long n_launch = 0;  // kernels launched by this context (all kinds)
-  bool per_op = true;      // one kernel per op (else the persistent single-launch forward)
+  bool per_op = false;     // one kernel per op instead of the persistent single-launch forward
   int fwd_grid = 0;
   unsigned int* fwd_bar = nullptr;
   unsigned long long* fwd_trace = nullptr;  // per-phase timestamps of the last forward (tracing on)
@@ -588,6 +588,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     f.err = c->err_word;
     f.trace = c->fwd_trace;
     CK(cudaMemsetAsync(c->fwd_bar, 0, sizeof(unsigned int), st));
+    CK(cudaMemsetAsync(m.att_counters, 0, (size_t)nqt * m.H * sizeof(int), st));
     if (c->fwd_trace) CK(cudaMemsetAsync(c->fwd_trace, 0, c->fwd_trace_n * sizeof(unsigned long long), st));
     const double wbytes = 2.0 * m.layers * (4.0 * m.d * m.d + 3.0 * m.d * m.ffn) + 2.0 * ITEM_ROWS * m.d;
     ProfScope ps(c, st, 6, wbytes, 2.0 * T * (wbytes / 2.0));
@@ -1203,9 +1204,9 @@ atspeed_status atspeed_create(const atspeed_model_desc* target, const atspeed_mo
     c->gemm_grid = gemm_grid_size(c->device);
     c->fwd_grid = c->gemm_grid;  // one persistent CTA per SM
     {
-      // ATSPEED_FORWARD=persistent selects the single-launch forward; the default is one kernel per op
+      // the forward runs as one persistent launch; ATSPEED_FORWARD=per_op selects one kernel per op
       const char* fm = getenv("ATSPEED_FORWARD");
-      c->per_op = !(fm && strcmp(fm, "persistent") == 0);
+      c->per_op = fm && strcmp(fm, "per_op") == 0;
     }
     c->fwd_bar = dalloc<unsigned int>(c, 1);
     {

@@ -36,12 +36,13 @@ __global__ void __launch_bounds__(128)
   attn_item<HD>(a, &mk, &mv, blockIdx.x, blockIdx.y, blockIdx.z, smem, bars, s_info, use, threadIdx.x, 1);
 }
 
-// One CTA of 128 threads per (query tile, head): merge the prefix splits with the path keys.
+// One CTA of 128 threads per (query tile, head, group of 16 queries): merge the prefix splits with
+// the path keys.
 template <int HD>
 __global__ void __launch_bounds__(128) attn_combine_kernel(const AttnArgs a) {
   pdl_launch_dependents();
   pdl_wait();
-  attn_combine_tile<HD>(a, blockIdx.x, blockIdx.y, threadIdx.x);
+  attn_combine_group<HD>(a, blockIdx.x, blockIdx.y, blockIdx.z, threadIdx.x);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn_att() {
@@ -79,7 +80,7 @@ cudaError_t launch_hd(const AttnArgs& a, const CUtensorMap& mk, const CUtensorMa
   cudaError_t e = cudaLaunchKernelEx(&cfg, attn_prefix_kernel<HD>, mk, mv, a);
   if (e != cudaSuccess || a.direct) return e;
   cudaLaunchConfig_t c2 = {};
-  c2.gridDim = dim3(a.n_qtiles, a.n_heads);
+  c2.gridDim = dim3(a.n_qtiles, a.n_heads, ATT_QTILE / ATT_CQ);
   c2.blockDim = dim3(128);
   c2.stream = st;
   c2.attrs = at;

@@ -313,60 +313,60 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
   return true;
 }
 
-// 128 threads: merge the prefix splits of every query of one (query tile, head) with the query's
-// path keys and write the normalised bf16 output.  Two threads per query, each owning half of the
-// head dimension; the dot products with the path keys add the two halves' fp32 partial sums in a
-// fixed order (lower half first), so the result does not depend on the schedule that calls it.
+// Queries per combine group: the merge of one (query tile, head) is split into ATT_QTILE / 16
+// groups of 16 queries, each handled by 128 threads (8 per query).
+constexpr int ATT_CQ = 16;
+
+// 128 threads: merge the prefix splits of 16 queries (group qg of the tile) of one head with each
+// query's path keys and write the normalised bf16 output.  Eight threads per query, each owning
+// HD / 8 consecutive dimensions; a path-key dot product adds the eight partial sums by a butterfly
+// over the eight lanes (exact in any lane, as fp32 addition commutes), so the result does not
+// depend on the schedule that calls it.
 template <int HD>
-__device__ void attn_combine_tile(const AttnArgs& a, int tile, int h, int ctid) {
-  constexpr int DH = HD / 2;
-  const int qi = ctid >> 1, half = ctid & 1;
+__device__ void attn_combine_group(const AttnArgs& a, int tile, int h, int qg, int ctid) {
+  constexpr int TPQ = 8, DH = HD / TPQ;
+  const int ql = qg * ATT_CQ + (ctid >> 3), part = ctid & 7;
   const int t0 = a.qt_t0[tile], nq = a.qt_n[tile];
-  const bool active = qi < nq;
-  const int t = t0 + (active ? qi : 0);
+  const bool active = ql < nq;
+  const int t = t0 + (active ? ql : 0);
   const int d = a.n_heads * HD;
   const int S = a.user_splits[a.qt_user[tile]];
   const float scale = kLog2e / sqrtf((float)HD);
-  const int dim0 = h * HD + half * DH;
+  const int dim0 = h * HD + part * DH;
+  // loads that do not depend on each other first: q, the path rows, the split statistics
   float qv[DH];
+  {
+    __nv_bfloat16 qb[DH];
 #pragma unroll
-  for (int i = 0; i < DH; i += 8) {
-    const uint4 r = __ldcg(reinterpret_cast<const uint4*>(a.q + (size_t)t * d + dim0 + i));
-    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&r);
+    for (int i = 0; i < DH; i += 4) *reinterpret_cast<uint2*>(qb + i) = __ldcg(reinterpret_cast<const uint2*>(a.q + (size_t)t * d + dim0 + i));
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float2 f = __bfloat1622float2(b[j]);
-      qv[i + 2 * j] = f.x;
-      qv[i + 2 * j + 1] = f.y;
-    }
+    for (int i = 0; i < DH; ++i) qv[i] = __bfloat162float(qb[i]);
   }
   const int na = (a.anc_n && active) ? a.anc_n[t] : 0;
-  float sa[ATT_MAX_ANC];
   int arow[ATT_MAX_ANC];
+#pragma unroll
+  for (int j = 0; j < ATT_MAX_ANC; ++j) arow[j] = j < na ? a.anc_row[t * ATT_MAX_ANC + j] : 0;
   float M = -INFINITY;
+  for (int s = 0; s < S; ++s) M = fmaxf(M, __ldcg(a.part_ml + (((size_t)s * a.T + t) * a.n_heads + h) * 2));
+  // path keys (rows written earlier in this forward; cached loads, queries share ancestors)
+  float sa[ATT_MAX_ANC];
 #pragma unroll
   for (int j = 0; j < ATT_MAX_ANC; ++j) {
-    float part = 0.f;
-    arow[j] = j < na ? a.anc_row[t * ATT_MAX_ANC + j] : 0;
+    float pd = 0.f;
     if (j < na) {
+      __nv_bfloat16 kb[DH];
 #pragma unroll
-      for (int i = 0; i < DH; i += 8) {
-        const uint4 r = __ldcg(reinterpret_cast<const uint4*>(a.k_cache + (size_t)arow[j] * d + dim0 + i));
-        const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&r);
+      for (int i = 0; i < DH; i += 4)
+        *reinterpret_cast<uint2*>(kb + i) = *reinterpret_cast<const uint2*>(a.k_cache + (size_t)arow[j] * d + dim0 + i);
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 f = __bfloat1622float2(b[e]);
-          part += qv[i + 2 * e] * f.x;
-          part += qv[i + 2 * e + 1] * f.y;
-        }
-      }
+      for (int i = 0; i < DH; ++i) pd += qv[i] * __bfloat162float(kb[i]);
     }
-    const float other = __shfl_xor_sync(0xffffffffu, part, 1);
-    const float dot = half == 0 ? part + other : other + part;
-    sa[j] = dot * scale;
+    pd += __shfl_xor_sync(0xffffffffu, pd, 1);
+    pd += __shfl_xor_sync(0xffffffffu, pd, 2);
+    pd += __shfl_xor_sync(0xffffffffu, pd, 4);
+    sa[j] = pd * scale;
     if (j < na) M = fmaxf(M, sa[j]);
   }
-  for (int s = 0; s < S; ++s) M = fmaxf(M, __ldcg(a.part_ml + (((size_t)s * a.T + t) * a.n_heads + h) * 2));
   const float Mu = (M == -INFINITY) ? 0.f : M;
   float L = 0.f, o[DH];
 #pragma unroll
@@ -374,16 +374,18 @@ __device__ void attn_combine_tile(const AttnArgs& a, int tile, int h, int ctid) 
   for (int s = 0; s < S; ++s) {
     const size_t b = ((size_t)s * a.T + t) * a.n_heads + h;
     const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.part_ml + b * 2));
+    const float* po = a.part_o + b * HD + part * DH;
+    float4 pv[DH / 4];
+#pragma unroll
+    for (int i = 0; i < DH; i += 4) pv[i / 4] = __ldcg(reinterpret_cast<const float4*>(po + i));
     const float w = exp2f(ml.x - Mu);
     L += ml.y * w;
-    const float* po = a.part_o + b * HD + half * DH;
 #pragma unroll
     for (int i = 0; i < DH; i += 4) {
-      const float4 v = __ldcg(reinterpret_cast<const float4*>(po + i));
-      o[i] += v.x * w;
-      o[i + 1] += v.y * w;
-      o[i + 2] += v.z * w;
-      o[i + 3] += v.w * w;
+      o[i] += pv[i / 4].x * w;
+      o[i + 1] += pv[i / 4].y * w;
+      o[i + 2] += pv[i / 4].z * w;
+      o[i + 3] += pv[i / 4].w * w;
     }
   }
 #pragma unroll
@@ -391,17 +393,12 @@ __device__ void attn_combine_tile(const AttnArgs& a, int tile, int h, int ctid) 
     if (j >= na) continue;
     const float w = exp2f(sa[j] - Mu);
     L += w;
+    __half vb[DH];
 #pragma unroll
-    for (int i = 0; i < DH; i += 8) {
-      const uint4 r = __ldcg(reinterpret_cast<const uint4*>(a.v_cache + (size_t)arow[j] * d + dim0 + i));
-      const __half2* hv = reinterpret_cast<const __half2*>(&r);
+    for (int i = 0; i < DH; i += 4)
+      *reinterpret_cast<uint2*>(vb + i) = *reinterpret_cast<const uint2*>(a.v_cache + (size_t)arow[j] * d + dim0 + i);
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 f = __half22float2(hv[e]);
-        o[i + 2 * e] += w * f.x;
-        o[i + 2 * e + 1] += w * f.y;
-      }
-    }
+    for (int i = 0; i < DH; ++i) o[i] += w * __half2float(vb[i]);
   }
   if (!active) return;
   const float inv = L > 0.f ? 1.f / L : 0.f;

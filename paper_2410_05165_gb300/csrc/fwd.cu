@@ -129,6 +129,21 @@ __device__ __forceinline__ void crange(const GP& g, int c, long long& u0, long l
   u1 = (long long)(c + 1) * g.U / g.Ge;
 }
 
+// Weight-tile coordinates of unit u: k offset and the rows of the two 64-row boxes (SwiGLU tiles
+// pair 64 gate rows with the matching 64 up rows).
+__device__ __forceinline__ void a_coords(const GP& g, long long u, int& x, int& y0, int& y1) {
+  const int tile = (int)(u / g.kb), kbi = (int)(u % g.kb);
+  const int mt = tile / g.n_tiles;
+  x = kbi * GEMM_BK;
+  if (g.epi == EPI_SWIGLU) {
+    y0 = mt * 64;
+    y1 = g.up_row0 + mt * 64;
+  } else {
+    y0 = mt * GEMM_BM;
+    y1 = mt * GEMM_BM + 64;
+  }
+}
+
 // phase index (in the compute warps' program) of GEMM phase gi
 __device__ __forceinline__ int gemm_phase_index(int gi, int L) {
   if (gi == 4 * L) return 1 + 7 * L;
@@ -182,6 +197,23 @@ __device__ bool cta_count_wait(const int* cnt, int target, unsigned* err) {
     __nanosleep(32);
     if (ld_acquire_cta(cnt) >= target) return true;
     if ((it & 1023u) == 0u) {
+      if (err_set(err)) return false;
+      if (globaltimer_ns() - t0 > kWaitBudgetNs) {
+        set_error(err, ATSPEED_DEV_ERR_TIMEOUT);
+        return false;
+      }
+    }
+  }
+}
+
+// Waits until the global counter reaches `target` (bounded; false on timeout or a raised error).
+__device__ bool counter_wait(const int* cnt, int target, unsigned* err) {
+  if ((int)ld_acquire_u32(reinterpret_cast<const unsigned*>(cnt)) >= target) return true;
+  const unsigned long long t0 = globaltimer_ns();
+  for (unsigned it = 1;; ++it) {
+    __nanosleep(64);
+    if ((int)ld_acquire_u32(reinterpret_cast<const unsigned*>(cnt)) >= target) return true;
+    if ((it & 255u) == 0u) {
       if (err_set(err)) return false;
       if (globaltimer_ns() - t0 > kWaitBudgetNs) {
         set_error(err, ATSPEED_DEV_ERR_TIMEOUT);
@@ -425,8 +457,8 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
   }
 }
 
-// Tree attention of layer l: this CTA's work items (query tile, head, prefix split); the last split
-// of a (tile, head) to finish merges the splits.
+// Tree attention of layer l: this CTA's work items (query tile, head, prefix split), each followed
+// by its share of the merge of the splits of (tile, head).
 template <int HD>
 __device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* att_smem, uint64_t* att_bars, int* s_info,
                                         int (&use_att)[2], int* flag, int ctid) {
@@ -449,19 +481,20 @@ __device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* a
     if (a.direct) continue;
     const int S_u = a.user_splits[a.qt_user[tile]];
     if (split >= S_u) continue;
+    // every split publishes its partials and waits for the others of (tile, h) -- they run in the
+    // same or a later round of items, never an earlier one -- then split s merges query groups
+    // s, s + S_u, ...  The counter only grows during a launch: layer l completes at S_u * (l + 1).
     __threadfence();
     named_bar_sync(1, 128);
     if (ctid == 0) {
-      const int old = atomicAdd(&p.att_counters[tile * H + h], 1);
-      const int last = old == S_u - 1;
-      if (last) {
-        p.att_counters[tile * H + h] = 0;
-        __threadfence();
-      }
-      *flag = last;
+      int* cnt = &p.att_counters[tile * H + h];
+      atomicAdd(cnt, 1);
+      *flag = counter_wait(cnt, S_u * (l + 1), p.err) ? 1 : 0;
     }
     named_bar_sync(1, 128);
-    if (*flag) attn_combine_tile<HD>(a, tile, h, ctid);
+    if (!*flag) return false;
+    const int nq = a.qt_n[tile];
+    for (int qg = split; qg * ATT_CQ < nq; qg += S_u) attn_combine_group<HD>(a, tile, h, qg, ctid);
     named_bar_sync(1, 128);
     if (p.trace && ctid == 0 && nit < 2) p.trace[((size_t)(5 + 2 * nit) * NP + ph) * G + c] = globaltimer_ns();
   }
@@ -703,21 +736,13 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
             ok = false;
             break;
           }
-          const int tile = (int)(u / g.kb), kbi = (int)(u % g.kb);
-          const int mt = tile / g.n_tiles;
-          int r0, r1;
-          if (g.epi == EPI_SWIGLU) {
-            r0 = mt * 64;
-            r1 = g.up_row0 + mt * 64;
-          } else {
-            r0 = mt * GEMM_BM;
-            r1 = mt * GEMM_BM + 64;
-          }
+          int kx, r0, r1;
+          a_coords(g, u, kx, r0, r1);
           uint8_t* sa = ringA + s * C::A_BYTES;
           mbar_arrive_expect_tx(&fullA[s], C::A_BYTES);
           lastA[s] = (int)ph;
-          tma_load_2d(sa, mA, &fullA[s], kbi * GEMM_BK, r0, pol);
-          tma_load_2d(sa + 8192, mA, &fullA[s], kbi * GEMM_BK, r1, pol);
+          tma_load_2d(sa, mA, &fullA[s], kx, r0, pol);
+          tma_load_2d(sa + 8192, mA, &fullA[s], kx, r1, pol);
         }
       }
       if (!ok) *failed = 1;

@@ -54,7 +54,7 @@ struct FwdParams {
   // attention (k_cache / v_cache of `att_args` are set per layer inside the kernel)
   AttnArgs att_args;
   int att_items;            // n_qtiles * H * max_splits
-  int* att_counters;        // [n_qtiles * H], zero, left zero
+  int* att_counters;        // [n_qtiles * H], zeroed before the launch (split arrivals, all layers)
   // GEMM split-K scratch
   float* ws;
   int* counters;            // zero, left zero
