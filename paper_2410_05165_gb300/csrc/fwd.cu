@@ -244,7 +244,6 @@ __device__ __noinline__ void epi_dispatch(int epi, const GemmArgs& a, const floa
                                              int t, const int* tpos, const int* tkvr) {
   switch (epi) {
     case EPI_F32: epi_chunk<BN, EPI_F32>(a, st, mt, nt, ch, t, tpos, tkvr); break;
-    case EPI_RESID: epi_chunk<BN, EPI_RESID>(a, st, mt, nt, ch, t, tpos, tkvr); break;
     case EPI_SWIGLU: epi_chunk<BN, EPI_SWIGLU>(a, st, mt, nt, ch, t, tpos, tkvr); break;
     default: epi_chunk<BN, EPI_QKV>(a, st, mt, nt, ch, t, tpos, tkvr); break;
   }
