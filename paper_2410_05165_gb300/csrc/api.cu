@@ -138,6 +138,8 @@ struct atspeed_ctx {
   bool per_op = false;     // one kernel per op instead of the persistent single-launch forward
   int fwd_grid = 0;
   unsigned int* fwd_bar = nullptr;
+  int* fwd_sk = nullptr;     // split-tile arrival counters of the persistent forward
+  size_t fwd_sk_n = 0;
   unsigned long long* fwd_trace = nullptr;  // per-phase timestamps of the last forward (tracing on)
   size_t fwd_trace_n = 0;
 };
@@ -584,11 +586,13 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     f.att_counters = m.att_counters;
     f.ws = c->gs.ws;
     f.counters = c->gs.counters;
+    f.sk_counters = c->fwd_sk;
     f.bar = c->fwd_bar;
     f.err = c->err_word;
     f.trace = c->fwd_trace;
     CK(cudaMemsetAsync(c->fwd_bar, 0, sizeof(unsigned int), st));
     CK(cudaMemsetAsync(m.att_counters, 0, (size_t)nqt * m.H * sizeof(int), st));
+    CK(cudaMemsetAsync(c->fwd_sk, 0, (size_t)(4 * m.layers + 1) * c->fwd_grid * sizeof(int), st));
     if (c->fwd_trace) CK(cudaMemsetAsync(c->fwd_trace, 0, c->fwd_trace_n * sizeof(unsigned long long), st));
     const double wbytes = 2.0 * m.layers * (4.0 * m.d * m.d + 3.0 * m.d * m.ffn) + 2.0 * ITEM_ROWS * m.d;
     ProfScope ps(c, st, 6, wbytes, 2.0 * T * (wbytes / 2.0));
@@ -1209,6 +1213,11 @@ atspeed_status atspeed_create(const atspeed_model_desc* target, const atspeed_mo
       c->per_op = fm && strcmp(fm, "per_op") == 0;
     }
     c->fwd_bar = dalloc<unsigned int>(c, 1);
+    {
+      const int Lmax = std::max(c->tgt.layers, c->drf.present ? c->drf.layers : 0);
+      c->fwd_sk_n = (size_t)(4 * Lmax + 1) * c->fwd_grid;
+      c->fwd_sk = dalloc<int>(c, c->fwd_sk_n);
+    }
     {
       const char* tr = getenv("ATSPEED_FWD_TRACE");
       if (tr && tr[0] == '1') {

@@ -63,8 +63,7 @@ struct GP {
   int epi;
   bool to_dh;    // O / down projection: the product goes to dh (the next norm phase adds it to h)
   int M, K, m_tiles, n_tiles, kb, up_row0, rows;  // rows: valid tokens of the phase
-  long long U;
-  int Ge;        // CTAs that receive units: min(G, U) (the others idle in this phase)
+  WorkSplit w;   // whole tiles per CTA + stream-K over the remaining tiles
   int mapA, mapB, layer;
 };
 
@@ -114,25 +113,13 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
   g.m_tiles = (g.epi == EPI_SWIGLU) ? g.M / GEMM_BM : (g.M + GEMM_BM - 1) / GEMM_BM;
   g.n_tiles = (g.rows + BN - 1) / BN;
   g.kb = g.K / GEMM_BK;
-  g.U = (long long)g.m_tiles * g.n_tiles * g.kb;
-  g.Ge = (int)((long long)p.G < g.U ? p.G : g.U);
+  g.w = work_split(g.m_tiles * g.n_tiles, g.kb, p.G);
   return g;
 }
 
-// This CTA's unit range [u0, u1) of a GEMM phase (same partition as the standalone GEMM).
-__device__ __forceinline__ void crange(const GP& g, int c, long long& u0, long long& u1) {
-  if (c >= g.Ge) {
-    u0 = u1 = 0;
-    return;
-  }
-  u0 = (long long)c * g.U / g.Ge;
-  u1 = (long long)(c + 1) * g.U / g.Ge;
-}
-
-// Weight-tile coordinates of unit u: k offset and the rows of the two 64-row boxes (SwiGLU tiles
-// pair 64 gate rows with the matching 64 up rows).
-__device__ __forceinline__ void a_coords(const GP& g, long long u, int& x, int& y0, int& y1) {
-  const int tile = (int)(u / g.kb), kbi = (int)(u % g.kb);
+// Weight-tile coordinates of (tile, k-block): k offset and the rows of the two 64-row boxes
+// (SwiGLU tiles pair 64 gate rows with the matching 64 up rows).
+__device__ __forceinline__ void a_coords(const GP& g, int tile, int kbi, int& x, int& y0, int& y1) {
   const int mt = tile / g.n_tiles;
   x = kbi * GEMM_BK;
   if (g.epi == EPI_SWIGLU) {
@@ -151,8 +138,6 @@ __device__ __forceinline__ int gemm_phase_index(int gi, int L) {
   return 7 * l + (k == 0 ? 1 : k == 1 ? 3 : k == 2 ? 5 : 6);
 }
 
-__device__ __forceinline__ long long ustart(long long c, long long U, int G) { return c * U / G; }
-__device__ __forceinline__ int uowner(long long u, long long U, int G) { return (int)(((u + 1) * (long long)G - 1) / U); }
 
 __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* a) {
   unsigned v;
@@ -289,9 +274,12 @@ __device__ void build_part_table(const FwdParams& p, int gi, int nt, int* toff, 
   int cnt = 0, c_first = 0;
   long long tu0 = 0;
   if (ctid < g.m_tiles) {
-    tu0 = (long long)(ctid * g.n_tiles + nt) * g.kb;
-    c_first = uowner(tu0, g.U, g.Ge);
-    cnt = uowner(tu0 + g.kb - 1, g.U, g.Ge) - c_first + 1;
+    const int t = ctid * g.n_tiles + nt;
+    if (t < g.w.r) {   // a stream-K tile; whole tiles have a single part, written to dh
+      tu0 = (long long)t * g.kb;
+      c_first = sk_owner(g.w, tu0);
+      cnt = sk_owner(g.w, tu0 + g.kb - 1) - c_first + 1;
+    }
     if (cnt == 1) cnt = 0;
     toff[ctid + 1] = cnt;
   }
@@ -305,7 +293,7 @@ __device__ void build_part_table(const FwdParams& p, int gi, int nt, int* toff, 
     for (int pi = 0; pi < cnt; ++pi) {
       const int cc = c_first + pi;
       const int e = toff[ctid] + pi;
-      if (e < PART_TABLE_CAP) tslot[e] = cc * 2 + (ustart(cc, g.U, g.Ge) >= tu0 ? 0 : 1);
+      if (e < PART_TABLE_CAP) tslot[e] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
     }
   }
   if (ctid == 0 && toff[g.m_tiles] > PART_TABLE_CAP) set_error(p.err, ATSPEED_DEV_ERR_BOUNDS);
@@ -518,15 +506,60 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
   const GP g = gemm_phase(p, gi, BN);
   const GemmArgs ea = epi_args(p, g);
   const int kb = g.kb;
-  long long u0, u1;
-  crange(g, c, u0, u1);
-  int seg = 0;
-  for (long long u = u0; u < u1; ++si, ++seg) {
-    const int tile = (int)(u / kb);
-    const int k0 = (int)(u % kb);
-    const long long len = (kb - k0) < (u1 - u) ? (kb - k0) : (u1 - u);
-    const int k1 = k0 + (int)len;
-    u += len;
+  SegIter it;
+  it.init(g.w, c);
+  int tile, k0, k1;
+  if (g.w.q > 0 && !g.to_dh && it.u < it.u1) {
+    // A phase with whole tiles per CTA: the split (stream-K) tiles come first and finish early.
+    // Every part publishes its partial sum (all of this CTA's, before any wait), then each part
+    // sums a share of its tile's chunks (chunk ch by part ch mod parts) -- spread over the parts'
+    // CTAs instead of one, while their whole tiles are still in the tensor pipe.
+    int sk_tile[2], nsk = 0;
+    while (it.u < it.u1 && nsk < 2) {
+      it.next(g.w, tile, k0, k1);
+      const int acc = si & 1, use = si >> 1;
+      ++si;
+      const bool got = mwait(&tfull[acc], (uint32_t)(use & 1), p.err);
+      __syncwarp();
+      if (!got) return false;
+      tc_fence_after();
+      const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+      const int nch = min(BN / 32, (g.rows - (tile % g.n_tiles) * BN + 31) / 32);
+      ws_store_partial(p.ws + ((long long)c * 2 + nsk) * GEMM_WS_SLOT_FLOATS, tb, nch, m);
+      tc_fence_before();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      sk_tile[nsk++] = tile;
+    }
+    __threadfence();
+    named_bar_sync(1, 128);
+    int* skc = p.sk_counters + (size_t)gi * G;
+    if (ctid == 0)
+      for (int j = 0; j < nsk; ++j) atomicAdd(&skc[sk_tile[j]], 1);
+    for (int j = 0; j < nsk; ++j) {
+      const int t = sk_tile[j];
+      const long long tu0 = (long long)t * kb;
+      const int c_first = sk_owner(g.w, tu0);
+      const int parts = sk_owner(g.w, tu0 + kb - 1) - c_first + 1;
+      const int m_tile = t / g.n_tiles, n_tile = t % g.n_tiles;
+      for (int pi = ctid; pi < parts; pi += 128) {
+        const int cc = c_first + pi;
+        part_slot[pi] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
+      }
+      if (g.epi == EPI_QKV) load_tok_tables<BN>(ea, n_tile, tpos, tkvr, ctid);
+      if (ctid == 0) *flag = counter_wait(&skc[t], parts, p.err) ? 1 : 0;
+      named_bar_sync(1, 128);
+      if (!*flag) return false;
+      const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
+      for (int ch = c - c_first; ch < nch; ch += parts) {
+        ws_reduce_chunk(p.ws, part_slot, parts, ch, m, staging);
+        named_bar_sync(1, 128);
+        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid, tpos, tkvr);
+        named_bar_sync(1, 128);
+      }
+      named_bar_sync(1, 128);   // flag, part_slot and the token tables are reused
+    }
+  }
+  for (int seg = 0; it.next(g.w, tile, k0, k1); ++si, ++seg) {
     const int acc = si & 1, use = si >> 1;
     const int m_tile = tile / g.n_tiles, n_tile = tile % g.n_tiles;
     const bool whole = (k0 == 0 && k1 == kb);
@@ -535,11 +568,11 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
     int c_first = 0, parts = 1;
     if (!whole && !g.to_dh) {
       tu0 = (long long)tile * kb;
-      c_first = uowner(tu0, g.U, g.Ge);
-      parts = uowner(tu0 + kb - 1, g.U, g.Ge) - c_first + 1;
+      c_first = sk_owner(g.w, tu0);
+      parts = sk_owner(g.w, tu0 + kb - 1) - c_first + 1;
       for (int pi = ctid; pi < parts; pi += 128) {
         const int cc = c_first + pi;
-        part_slot[pi] = cc * 2 + (ustart(cc, g.U, g.Ge) >= tu0 ? 0 : 1);
+        part_slot[pi] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
       }
     }
     const bool got = mwait(&tfull[acc], (uint32_t)(use & 1), p.err);
@@ -590,8 +623,11 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       if (lane == 0) mbar_arrive(&tempty[acc]);
       continue;
     }
-    // split tile: are the other parts all published already?
-    if (ctid == 0) *flag = (int)ld_acquire_u32(reinterpret_cast<const unsigned*>(&p.counters[tile])) == parts - 1;
+    // split tile: are the other parts all published already?  (Only for the CTA's last segment of
+    // the phase: holding this accumulator through the sum must not stall later MMAs of the phase.)
+    if (ctid == 0)
+      *flag = !it.more() &&
+              (int)ld_acquire_u32(reinterpret_cast<const unsigned*>(&p.counters[tile])) == parts - 1;
     named_bar_sync(1, 128);
     if (*flag) {
       // last part: nobody else touches this tile's counter in this phase
@@ -726,22 +762,25 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
       for (int gi = 0; gi < NG && ok; ++gi) {
         const GP g = gemm_phase(p, gi, BN);
         const CUtensorMap* mA = p.maps + g.mapA;
-        long long u0, u1;
-        crange(g, c, u0, u1);
-        for (long long u = u0; u < u1; ++u, ++n) {
-          const int s = (int)(n % C::SA);
-          const uint32_t ph = (uint32_t)((n / C::SA) & 1);
-          if (!mwait(&emptyA[s], ph ^ 1u, p.err)) {
-            ok = false;
-            break;
-          }
+        SegIter it;
+        it.init(g.w, c);
+        int tile, k0, k1;
+        while (ok && it.next(g.w, tile, k0, k1)) {
           int kx, r0, r1;
-          a_coords(g, u, kx, r0, r1);
-          uint8_t* sa = ringA + s * C::A_BYTES;
-          mbar_arrive_expect_tx(&fullA[s], C::A_BYTES);
-          lastA[s] = (int)ph;
-          tma_load_2d(sa, mA, &fullA[s], kx, r0, pol);
-          tma_load_2d(sa + 8192, mA, &fullA[s], kx, r1, pol);
+          a_coords(g, tile, k0, kx, r0, r1);
+          for (int kbi = k0; kbi < k1; ++kbi, ++n, kx += GEMM_BK) {
+            const int s = (int)(n % C::SA);
+            const uint32_t ph = (uint32_t)((n / C::SA) & 1);
+            if (!mwait(&emptyA[s], ph ^ 1u, p.err)) {
+              ok = false;
+              break;
+            }
+            uint8_t* sa = ringA + s * C::A_BYTES;
+            mbar_arrive_expect_tx(&fullA[s], C::A_BYTES);
+            lastA[s] = (int)ph;
+            tma_load_2d(sa, mA, &fullA[s], kx, r0, pol);
+            tma_load_2d(sa + 8192, mA, &fullA[s], kx, r1, pol);
+          }
         }
       }
       if (!ok) *failed = 1;
@@ -754,30 +793,33 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
       bool ok = true;
       for (int gi = 0; gi < NG && ok; ++gi) {
         const GP g = gemm_phase(p, gi, BN);
-        long long u0, u1;
-        crange(g, c, u0, u1);
+        const long long nu = cta_units(g.w, c);
         // the compute warps pass the grid barrier that publishes this phase's input and count it in
         // `go` (one grid poller per CTA)
         if (!cta_count_wait(go, gi + 1, p.err)) {
           ok = false;
           break;
         }
-        if (u1 <= u0) continue;
+        if (nu == 0) continue;
         if (p.trace) p.trace[((size_t)1 * (7 * L + 2) + gi) * G + c] = globaltimer_ns();
         fence_proxy_async();
         const CUtensorMap* mB = p.maps + g.mapB;
-        for (long long u = u0; u < u1; ++u, ++n) {
-          const int s = (int)(n % C::SB);
-          const uint32_t ph = (uint32_t)((n / C::SB) & 1);
-          if (!mwait(&emptyB[s], ph ^ 1u, p.err)) {
-            ok = false;
-            break;
-          }
-          const int tile = (int)(u / g.kb), kbi = (int)(u % g.kb);
+        SegIter it;
+        it.init(g.w, c);
+        int tile, k0, k1;
+        while (ok && it.next(g.w, tile, k0, k1)) {
           const int nt = tile % g.n_tiles;
-          mbar_arrive_expect_tx(&fullB[s], C::B_BYTES);
-          lastB[s] = (int)ph;
-          tma_load_2d(ringB + s * C::B_BYTES, mB, &fullB[s], kbi * GEMM_BK, nt * BN, pol);
+          for (int kbi = k0; kbi < k1; ++kbi, ++n) {
+            const int s = (int)(n % C::SB);
+            const uint32_t ph = (uint32_t)((n / C::SB) & 1);
+            if (!mwait(&emptyB[s], ph ^ 1u, p.err)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&fullB[s], C::B_BYTES);
+            lastB[s] = (int)ph;
+            tma_load_2d(ringB + s * C::B_BYTES, mB, &fullB[s], kbi * GEMM_BK, nt * BN, pol);
+          }
         }
         if (p.trace) p.trace[((size_t)2 * (7 * L + 2) + gi) * G + c] = globaltimer_ns();
       }
@@ -793,13 +835,15 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
       bool ok = true;
       for (int gi = 0; gi < NG && ok; ++gi) {
         const GP g = gemm_phase(p, gi, BN);
-        long long u0, u1;
-        crange(g, c, u0, u1);
-        for (long long u = u0; u < u1 && ok; ++si) {
-          const int k0 = (int)(u % g.kb);
-          const long long len = (g.kb - k0) < (u1 - u) ? (g.kb - k0) : (u1 - u);
-          u += len;
+        SegIter it;
+        it.init(g.w, c);
+        int tile, k0, k1;
+        bool any = false;
+        while (ok && it.next(g.w, tile, k0, k1)) {
+          any = true;
+          const long long len = k1 - k0;
           const int acc = si & 1, use = si >> 1;
+          ++si;
           if (!mwait(&tempty[acc], (uint32_t)(use & 1) ^ 1u, p.err)) {
             ok = false;
             break;
@@ -825,7 +869,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
           if (!ok) break;
           tc_commit(&tfull[acc]);
         }
-        if (p.trace && u1 > u0) {
+        if (p.trace && any) {
           // time the last MMA of this phase completed
           tc_commit(mma_done);
           mbar_wait(mma_done, (uint32_t)(mma_waits & 1), nullptr);

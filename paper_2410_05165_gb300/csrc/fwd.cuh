@@ -58,6 +58,8 @@ struct FwdParams {
   // GEMM split-K scratch
   float* ws;
   int* counters;            // zero, left zero
+  int* sk_counters;         // [GEMM phases][G] split-tile arrivals of phases with whole tiles per CTA,
+                            // zeroed before the launch
   // grid barrier: monotonic arrival counter, zeroed before the launch
   unsigned int* bar;
   unsigned int* err;

@@ -44,7 +44,7 @@ struct Cfg {
 struct KParams {
   GemmArgs a;
   int m_tiles, n_tiles, kb;
-  long long U;
+  WorkSplit w;   // whole tiles per CTA + stream-K over the remaining tiles
   int G;
   int up_row0;
   float* ws;
@@ -52,10 +52,6 @@ struct KParams {
   unsigned int* err;
 };
 
-__device__ __forceinline__ long long unit_start(long long c, long long U, int G) { return c * U / G; }
-__device__ __forceinline__ int unit_owner(long long u, long long U, int G) {
-  return (int)(((u + 1) * (long long)G - 1) / U);
-}
 
 template <int BN, int EPI>
 __global__ void __launch_bounds__(192, 1)
@@ -80,7 +76,7 @@ __global__ void __launch_bounds__(192, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x;
-  const long long u0 = unit_start(c, p.U, p.G), u1 = unit_start(c + 1, p.U, p.G);
+  const long long nu = cta_units(p.w, c);   // this CTA's units (stream-K units, then whole tiles)
   const int kb = p.kb;
 
   if (threadIdx.x == 0) {
@@ -108,16 +104,21 @@ __global__ void __launch_bounds__(192, 1)
   pdl_launch_dependents();
 
   if (warp == 0) {
-    if (lane == 0 && u1 > u0) {
+    if (lane == 0 && nu > 0) {
       // ------------------------------------------------------------------ TMA producer
       tma_prefetch_desc(&tmA);
       tma_prefetch_desc(&tmB);
       const uint64_t pol_w = policy_evict_first();   // weights: streamed once
       const uint64_t pol_x = policy_evict_last();    // activations: re-read by every CTA
-      const long long total = u1 - u0;
+      const long long total = nu;
       const int npre = (int)(total < C::STAGES ? total : C::STAGES);
-      auto a_rows = [&](long long u, int& r0, int& r1, int& xk, int& brow) {
-        const int tile = (int)(u / kb), kbi = (int)(u % kb);
+      // units in order, walked segment by segment (no per-unit divisions)
+      SegIter it;
+      it.init(p.w, c);
+      int cur_tile = 0, cur_k = 0, cur_k1 = 0;
+      auto a_rows = [&](int& r0, int& r1, int& xk, int& brow) {
+        if (cur_k >= cur_k1) it.next(p.w, cur_tile, cur_k, cur_k1);
+        const int tile = cur_tile, kbi = cur_k++;
         const int mt = tile / p.n_tiles, nt = tile % p.n_tiles;
         if (EPI == EPI_SWIGLU) {
           r0 = mt * 64;
@@ -130,21 +131,19 @@ __global__ void __launch_bounds__(192, 1)
         brow = nt * BN;
       };
       // prologue: weights do not depend on the previous kernel, so fetch them before waiting
+      int pre_xk[C::STAGES], pre_brow[C::STAGES];
       for (int i = 0; i < npre; ++i) {
-        int r0, r1, xk, brow;
-        a_rows(u0 + i, r0, r1, xk, brow);
+        int r0, r1;
+        a_rows(r0, r1, pre_xk[i], pre_brow[i]);
         uint8_t* sa = smem + i * C::STAGE_BYTES;
         mbar_arrive_expect_tx(&full[i], C::STAGE_BYTES);
         last_fill[i] = 0;
-        tma_load_2d(sa, &tmA, &full[i], xk, r0, pol_w);
-        tma_load_2d(sa + 8192, &tmA, &full[i], xk, r1, pol_w);
+        tma_load_2d(sa, &tmA, &full[i], pre_xk[i], r0, pol_w);
+        tma_load_2d(sa + 8192, &tmA, &full[i], pre_xk[i], r1, pol_w);
       }
       pdl_wait();
-      for (int i = 0; i < npre; ++i) {
-        int r0, r1, xk, brow;
-        a_rows(u0 + i, r0, r1, xk, brow);
-        tma_load_2d(smem + i * C::STAGE_BYTES + C::A_BYTES, &tmB, &full[i], xk, brow, pol_x);
-      }
+      for (int i = 0; i < npre; ++i)
+        tma_load_2d(smem + i * C::STAGE_BYTES + C::A_BYTES, &tmB, &full[i], pre_xk[i], pre_brow[i], pol_x);
       int stage = npre % C::STAGES;
       uint32_t phase = (npre == C::STAGES) ? 1u : 0u;
       for (long long i = npre; i < total; ++i) {
@@ -153,7 +152,7 @@ __global__ void __launch_bounds__(192, 1)
           break;
         }
         int r0, r1, xk, brow;
-        a_rows(u0 + i, r0, r1, xk, brow);
+        a_rows(r0, r1, xk, brow);
         uint8_t* sa = smem + stage * C::STAGE_BYTES;
         mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
         last_fill[stage] = (int)phase;
@@ -167,17 +166,18 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0 && u1 > u0) {
+    if (lane == 0 && nu > 0) {
       // ------------------------------------------------------------------ MMA issuer
       constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
       int stage = 0;
       uint32_t phase = 0;
       int si = 0;
       bool ok = true;
-      for (long long u = u0; u < u1 && ok; ++si) {
-        const int k0 = (int)(u % kb);
-        const long long len = (kb - k0) < (u1 - u) ? (kb - k0) : (u1 - u);
-        u += len;
+      SegIter it;
+      it.init(p.w, c);
+      int tile, k0, k1;
+      for (; ok && it.next(p.w, tile, k0, k1); ++si) {
+        const long long len = k1 - k0;
         const int acc = si & 1, use = si >> 1;
         if (!mbar_wait(&tempty[acc], (uint32_t)(use & 1) ^ 1u, p.err)) {
           ok = false;
@@ -220,12 +220,10 @@ __global__ void __launch_bounds__(192, 1)
     const int m = q * 32 + lane;
     pdl_wait();
     int si = 0;
-    for (long long u = u0; u < u1; ++si) {
-      const int tile = (int)(u / kb);
-      const int k0 = (int)(u % kb);
-      const long long len = (kb - k0) < (u1 - u) ? (kb - k0) : (u1 - u);
-      const int k1 = k0 + (int)len;
-      u += len;
+    SegIter it;
+    it.init(p.w, c);
+    int tile, k0, k1;
+    for (; it.next(p.w, tile, k0, k1); ++si) {
       const int acc = si & 1, use = si >> 1;
       const bool got = mbar_wait(&tfull[acc], (uint32_t)(use & 1), p.err);
       __syncwarp();
@@ -260,8 +258,8 @@ __global__ void __launch_bounds__(192, 1)
         __threadfence();
         named_bar_sync(1, 128);
         const long long tu0 = (long long)tile * kb;
-        const int c_first = unit_owner(tu0, p.U, p.G);
-        const int c_last = unit_owner(tu0 + kb - 1, p.U, p.G);
+        const int c_first = sk_owner(p.w, tu0);
+        const int c_last = sk_owner(p.w, tu0 + kb - 1);
         const int parts = c_last - c_first + 1;
         if (ep_tid == 0) {
           const int old = atomicAdd(&p.counters[tile], 1);
@@ -275,7 +273,7 @@ __global__ void __launch_bounds__(192, 1)
         // workspace slot of every part, in k order
         for (int pi = ep_tid; pi < parts; pi += 128) {
           const int cc = c_first + pi;
-          part_slot[pi] = cc * 2 + (unit_start(cc, p.U, p.G) >= tu0 ? 0 : 1);
+          part_slot[pi] = cc * 2 + (sk_start(p.w, cc) >= tu0 ? 0 : 1);
         }
         named_bar_sync(1, 128);
         if (*flag) {
@@ -419,8 +417,9 @@ cudaError_t gemm_launch(const GemmArgs& a, const GemmScratch& s, int grid, cudaS
     snprintf(eb, el, "gemm: %lld tiles exceed the counter table (%d)", tiles, s.max_tiles);
     return cudaErrorInvalidValue;
   }
-  kp.U = tiles * kp.kb;
-  kp.G = (int)((long long)grid < kp.U ? grid : kp.U);
+  const long long U = tiles * kp.kb;
+  kp.G = (int)((long long)grid < U ? grid : U);
+  kp.w = work_split((int)tiles, kp.kb, kp.G);
   if (s.ws_bytes < gemm_ws_bytes(kp.G)) {
     snprintf(eb, el, "gemm: workspace too small");
     return cudaErrorInvalidValue;

@@ -9,6 +9,90 @@ constexpr int GEMM_BK = 64;    // bf16 elements per 128-byte swizzle row (one k-
 constexpr int GEMM_BM = 128;   // weight rows per tile (MMA M)
 constexpr int GEMM_WS_SLOT_FLOATS = 256 * 128;
 
+// ---- work split of a tiled GEMM over G CTAs (tiles of kb k-blocks)
+// Each CTA takes q = tiles / G whole tiles; the first r = tiles % G tiles are split by k-blocks into
+// G equal contiguous unit ranges (stream-K; unit = one tile's k-block).  A CTA works on its
+// stream-K units first and then on its whole tiles r + c q ... r + c q + q - 1, so the partial sums
+// of the split tiles are published early and the tail after the last MMA is whole-tile epilogues.
+// With tiles < G (q = 0) this is plain stream-K over all tiles.
+struct WorkSplit {
+  int tiles, kb, q, r;
+  long long Usk;   // stream-K units: r * kb
+  int Gsk;         // CTAs that get stream-K units: min(G, Usk)
+};
+
+__host__ __device__ inline WorkSplit work_split(int tiles, int kb, int G) {
+  WorkSplit w;
+  w.tiles = tiles;
+  w.kb = kb;
+  w.q = tiles / G;
+  w.r = tiles - w.q * G;
+  w.Usk = (long long)w.r * kb;
+  w.Gsk = (int)(w.Usk < (long long)G ? w.Usk : (long long)G);
+  return w;
+}
+// stream-K unit range [a, b) of CTA c
+__device__ __forceinline__ void sk_range(const WorkSplit& w, int c, long long& a, long long& b) {
+  if (c >= w.Gsk) {
+    a = b = 0;
+    return;
+  }
+  a = (long long)c * w.Usk / w.Gsk;
+  b = (long long)(c + 1) * w.Usk / w.Gsk;
+}
+__device__ __forceinline__ long long sk_start(const WorkSplit& w, long long c) { return c * w.Usk / w.Gsk; }
+__device__ __forceinline__ int sk_owner(const WorkSplit& w, long long u) {
+  return (int)(((u + 1) * (long long)w.Gsk - 1) / w.Usk);
+}
+// number of units of CTA c, and its i-th unit as (tile, k-block)
+__device__ __forceinline__ long long cta_units(const WorkSplit& w, int c) {
+  long long a, b;
+  sk_range(w, c, a, b);
+  return (b - a) + (long long)w.q * w.kb;
+}
+__device__ __forceinline__ void cta_unit(const WorkSplit& w, int c, long long i, int& tile, int& kbi) {
+  long long a, b;
+  sk_range(w, c, a, b);
+  if (i < b - a) {
+    const long long u = a + i;
+    tile = (int)(u / w.kb);
+    kbi = (int)(u - (long long)tile * w.kb);
+  } else {
+    const long long j = i - (b - a);
+    const int t = (int)(j / w.kb);
+    tile = w.r + c * w.q + t;
+    kbi = (int)(j - (long long)t * w.kb);
+  }
+}
+// the segments (one tile's contiguous k-blocks [k0, k1)) of CTA c in order
+struct SegIter {
+  long long u, u1;
+  int dp, dp1;
+  __device__ __forceinline__ void init(const WorkSplit& w, int c) {
+    sk_range(w, c, u, u1);
+    dp = w.r + c * w.q;
+    dp1 = dp + w.q;
+  }
+  __device__ __forceinline__ bool next(const WorkSplit& w, int& tile, int& k0, int& k1) {
+    if (u < u1) {
+      tile = (int)(u / w.kb);
+      k0 = (int)(u - (long long)tile * w.kb);
+      const long long len = (w.kb - k0) < (u1 - u) ? (w.kb - k0) : (u1 - u);
+      k1 = k0 + (int)len;
+      u += len;
+      return true;
+    }
+    if (dp < dp1) {
+      tile = dp++;
+      k0 = 0;
+      k1 = w.kb;
+      return true;
+    }
+    return false;
+  }
+  __device__ __forceinline__ bool more() const { return u < u1 || dp < dp1; }
+};
+
 // Per-token data of the QKV epilogue for the BN tokens of n-tile n_tile (rotary position and cache
 // row), copied to shared memory when a segment starts so that the epilogue's loads do not wait on
 // them.  Callers synchronise the 128 threads before the first chunk's epilogue.
