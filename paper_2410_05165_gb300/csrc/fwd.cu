@@ -509,11 +509,13 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
   SegIter it;
   it.init(g.w, c);
   int tile, k0, k1;
-  if (g.w.q > 0 && !g.to_dh && it.u < it.u1) {
-    // A phase with whole tiles per CTA: the split (stream-K) tiles come first and finish early.
-    // Every part publishes its partial sum (all of this CTA's, before any wait), then each part
-    // sums a share of its tile's chunks (chunk ch by part ch mod parts) -- spread over the parts'
-    // CTAs instead of one, while their whole tiles are still in the tensor pipe.
+  // Shared sums: in a phase with whole tiles per CTA the split (stream-K) tiles come first and
+  // finish early; in the LM head every tile is split into many short parts (and no CTA has more
+  // than two segments).  Every part publishes its partial sum (all of this CTA's, before any wait),
+  // then each part sums a share of its tile's chunks (chunk ch by part ch mod parts) -- spread over
+  // the parts' CTAs instead of one.
+  const bool shared_sums = !g.to_dh && (g.w.q > 0 || (gi == 4 * p.L && g.w.Gsk > 0 && g.w.Usk / g.w.Gsk + 1 < kb));
+  if (shared_sums && it.u < it.u1) {
     int sk_tile[2], nsk = 0;
     while (it.u < it.u1 && nsk < 2) {
       it.next(g.w, tile, k0, k1);
