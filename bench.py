@@ -34,6 +34,30 @@ import synth  # noqa: E402
 METRIC = "rec lists/sec (7B-shape target, K=10); verify-call % of HBM roofline"
 
 
+# ---- multi-rank host logic (replicas: every rank decodes its own users, nothing is exchanged on
+# the data path; only the timing is reduced)
+def shard_users(all_prompts, rank, world):
+    """This rank's users: an equal contiguous share of the job's users."""
+    n = len(all_prompts) // world
+    return all_prompts[rank * n:(rank + 1) * n]
+
+
+def job_ms(ms, world, device=None):
+    """Duration of the job's timed region: the slowest rank's (max over ranks)."""
+    if world == 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(users_per_rank, world, steps, ms):
+    """Whole-job throughput: the users of all ranks, steps lists each, over the job's duration."""
+    return users_per_rank * world * steps / (ms / 1e3)
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -204,8 +228,7 @@ def run_ours(args, w):
         return out
     tw, dw = to_dev(w.target, "target"), to_dev(w.draft, "draft")
     items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
-    prompts = synth.make_prompts(w.n_users * world, w.prompt_len, w.target.vocab, w.seed)[
-        rank * w.n_users:(rank + 1) * w.n_users]
+    prompts = shard_users(synth.make_prompts(w.n_users * world, w.prompt_len, w.target.vocab, w.seed), rank, world)
     B = len(prompts)
     P_users = [len(p) for p in prompts]
     ctx = ats.Context(w.target, tw, w.draft, dw, items, w.code_base, max_users=B, max_prompt=max(P_users),
@@ -237,12 +260,8 @@ def run_ours(args, w):
     barrier()
     clk = clocks.stop()
     launches = (ctx.profile_read(-1)["launches"] - l0) / args.steps
-    ms = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = B * world * args.steps / (ms / 1e3)
+    ms = job_ms(e0.elapsed_time(e1), world, "cuda")
+    value = job_rate(B, world, args.steps, ms)
 
     # ---- end to end through the C ABI: pinned host prompt -> device, decode, items -> host
     h_items = torch.empty(B, w.K, 4, dtype=torch.int32).pin_memory()
@@ -258,12 +277,8 @@ def run_ours(args, w):
         h_sc.copy_(d_sc, non_blocking=True)
     e1.record(stream)
     barrier()
-    ms_e2e = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([ms_e2e], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_e2e = float(t.item())
-    e2e = {"value": B * world * args.steps / (ms_e2e / 1e3), "unit": "rec lists/s",
+    ms_e2e = job_ms(e0.elapsed_time(e1), world, "cuda")
+    e2e = {"value": job_rate(B, world, args.steps, ms_e2e), "unit": "rec lists/s",
            "h2d_bytes_per_step": int(h_tok.numel() * 4), "d2h_bytes_per_step": int(h_items.numel() * 4 + h_sc.numel() * 4)}
 
     # ---- the verification call alone (first call of a decode: depth 0, T = 3 N tree tokens)
