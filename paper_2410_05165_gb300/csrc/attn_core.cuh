@@ -55,12 +55,14 @@ __device__ __forceinline__ uint32_t kv_off(int row, int chunk16) {
 
 template <int HD>
 struct AttCfg {
-  // SMEM_BODY: bytes from the 1024-aligned base (K/V double buffer, then the Q tile)
+  // SMEM_BODY: bytes from the 1024-aligned base: the K/V double buffer; the Q tile is staged in the
+  // second buffer before its first K/V copy (Q lives in registers from then on)
   static constexpr int QSTRIDE = HD + 8;                    // bf16 elements per Q row in smem
   static constexpr int Q_BYTES = ATT_QTILE * QSTRIDE * 2;
   static constexpr int KV_BYTES = ATT_PAGE * HD * 2;         // one K (or V) page tile
   static constexpr int BUF_BYTES = 2 * KV_BYTES;             // K + V
-  static constexpr int SMEM_BODY = 2 * BUF_BYTES + Q_BYTES;
+  static constexpr int SMEM_BODY = 2 * BUF_BYTES;
+  static_assert(Q_BYTES <= BUF_BYTES, "the Q tile must fit in one K/V buffer");
   static constexpr int SMEM = 1024 + SMEM_BODY + 64;
 };
 
@@ -78,7 +80,7 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
   constexpr int NDT = HD / 8;    // dim n-tiles of O
   constexpr int NKS = HD / 16;   // k-steps of Q K^T
   uint8_t* kvbuf = smem;                                             // [2][K | V]
-  __nv_bfloat16* qs = reinterpret_cast<__nv_bfloat16*>(smem + 2 * C::BUF_BYTES);
+  __nv_bfloat16* qs = reinterpret_cast<__nv_bfloat16*>(smem + C::BUF_BYTES);   // buffer 1, until chunk 2's copy
   const int warp = tid >> 5, lane = tid & 31;
   const int d = a.n_heads * HD;
   const int u = a.qt_user[tile];
@@ -162,6 +164,7 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
     for (int kk = 0; kk < NKS; ++kk)
       ldsm_x4(qbase + (uint32_t)((r * C::QSTRIDE + kk * 16 + cofs) * 2), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
   }
+  named_bar_sync(bar_id, 128);   // every warp holds its Q fragments: buffer 1 may receive K/V now
   const int g = lane >> 2, tq = lane & 3;
   const int row_a = warp * 16 + g, row_b = row_a + 8;
   const int vis_a = row_a < nq ? a.tok_vis[t0 + row_a] : 0;
@@ -177,8 +180,7 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
   for (int chunk = c0; chunk < c1; ++chunk) {
     const int buf = (chunk - c0) & 1;
     if (tid == 0 && chunk + 1 < c1) issue(chunk + 1, buf ^ 1);
-    const bool got = mbar_wait(&bars[buf], (uint32_t)(use[buf] & 1), a.err);
-    __syncwarp();
+    const bool got = named_bar_and(bar_id, 128, mbar_wait(&bars[buf], (uint32_t)(use[buf] & 1), a.err));
     if (chunk - c0 < 2) ATT_TR(2 + 2 * (chunk - c0));
     ++use[buf];
     if (!got) {

@@ -28,8 +28,9 @@ namespace atspeed {
 
 namespace {
 
-constexpr int FWD_THREADS = 256;
+constexpr int FWD_THREADS = 384;   // warps 0-3: producers, MMA; warps 4-11: two compute warpgroups
 constexpr int COMPUTE_WARP0 = 4;
+constexpr int CT = 256;            // compute threads (named barrier 1); warpgroup w uses barrier 2 + w
 constexpr int ITEM_ROWS_FWD = 1024;   // item-code rows of the LM head (4 levels x 256 codes)
 
 template <int BN>
@@ -38,7 +39,7 @@ struct FCfg {
   static constexpr int SB = BN == 128 ? 3 : 3;   // activation stages
   static constexpr int A_BYTES = GEMM_BM * 128;
   static constexpr int B_BYTES = BN * 128;
-  static constexpr int STAGING = 32 * GEMM_BM * 4;
+  static constexpr int STAGING = 2 * 32 * GEMM_BM * 4;   // one [32][128] fp32 chunk per warpgroup
   static constexpr int MISC = 8192;
   static constexpr int TMEM_COLS = 2 * BN;
 };
@@ -49,9 +50,11 @@ struct FLayout {
   static constexpr int A_OFF = 0;
   static constexpr int B_OFF = C::SA * C::A_BYTES;
   static constexpr int STG_OFF = B_OFF + C::SB * C::B_BYTES;
-  // the attention work area overlaps the activation ring and the staging buffer (both idle then)
+  // the attention work areas (one per warpgroup) overlap the activation ring and the staging buffers
+  // (both idle then)
   static constexpr int ATT_OFF = B_OFF;
-  static constexpr int ATT_NEED = AttCfg<HD>::SMEM_BODY;
+  static constexpr int ATT_BODY = ((AttCfg<HD>::SMEM_BODY + 1023) / 1024) * 1024;
+  static constexpr int ATT_NEED = 2 * ATT_BODY;
   static constexpr int AFTER_STG = STG_OFF + C::STAGING;
   static constexpr int EXTRA = (ATT_OFF + ATT_NEED > AFTER_STG) ? ((ATT_OFF + ATT_NEED - AFTER_STG + 1023) / 1024) * 1024 : 0;
   static constexpr int MISC_OFF = AFTER_STG + EXTRA;
@@ -270,7 +273,7 @@ constexpr int PART_TABLE_CAP = 512;
 template <int BN>
 __device__ void build_part_table(const FwdParams& p, int gi, int nt, int* toff, int* tslot, int ctid) {
   const GP g = gemm_phase(p, gi, BN);
-  named_bar_sync(1, 128);   // earlier readers of the table are done
+  named_bar_sync(1, CT);   // earlier readers of the table are done
   int cnt = 0, c_first = 0;
   long long tu0 = 0;
   if (ctid < g.m_tiles) {
@@ -283,12 +286,12 @@ __device__ void build_part_table(const FwdParams& p, int gi, int nt, int* toff, 
     if (cnt == 1) cnt = 0;
     toff[ctid + 1] = cnt;
   }
-  named_bar_sync(1, 128);
+  named_bar_sync(1, CT);
   if (ctid == 0) {
     toff[0] = 0;
     for (int t = 1; t <= g.m_tiles; ++t) toff[t] += toff[t - 1];
   }
-  named_bar_sync(1, 128);
+  named_bar_sync(1, CT);
   if (ctid < g.m_tiles) {
     for (int pi = 0; pi < cnt; ++pi) {
       const int cc = c_first + pi;
@@ -297,58 +300,52 @@ __device__ void build_part_table(const FwdParams& p, int gi, int nt, int* toff, 
     }
   }
   if (ctid == 0 && toff[g.m_tiles] > PART_TABLE_CAP) set_error(p.err, ATSPEED_DEV_ERR_BOUNDS);
-  named_bar_sync(1, 128);
+  named_bar_sync(1, CT);
 }
 
-// RMSNorm of rows (128 compute threads).  mode 0 = embedding gather + norm (layer 0); 1 = residual
-// add h += (product of the preceding O / down projection gi_prev, summed from its parts in k order
-// starting from zero), then norm of h; 2 = the same for the selected rows only (final norm).  The
-// sum of squares runs over two virtual threads per thread in the order of the 256-thread kernels,
-// so the result is the same, bit for bit.  Between the passes the row is kept in shared memory
-// (`rowbuf`, d floats: the activation ring, idle during a norm phase).
-constexpr int NORM_NB = 4;   // float4 chunks per virtual thread in flight
+// RMSNorm of rows (256 compute threads; the per-thread chunks and the reduction are those of the
+// 256-thread kernels, so the sums are the same bit for bit).  mode 0 = embedding gather + norm
+// (layer 0); 1 = residual add h += (product of the preceding O / down projection gi_prev, summed
+// from its parts in k order starting from zero), then norm of h; 2 = the same for the selected rows
+// only (final norm).  Between the passes the row is kept in shared memory (`rowbuf`, d floats: the
+// activation ring, idle during a norm phase).
+constexpr int NORM_NB = 4;   // float4 chunks per thread in flight
 
 template <int BN>
 __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const __nv_bfloat16* g, float* red,
-                                        float4* rowbuf, int ctid, int gi_prev, int* toff, int* tslot, int& tab_nt,
-                                        int ph) {
+                                           float4* rowbuf, int ctid, int gi_prev, int* toff, int* tslot,
+                                           int& tab_nt, int ph) {
   const int rows = mode == 2 ? p.n_out : p.T;
   const int d = p.d, nc = d / 4;
   const int w = ctid >> 5, lane = ctid & 31;
   for (int r = blockIdx.x; r < rows; r += p.G) {
     const int src = mode == 2 ? p.out_rows[r] : r;
     float* hr = p.h + (size_t)src * d;
-    float ss[2] = {0.f, 0.f};
+    float ss = 0.f;
     if (mode == 0) {
       const __nv_bfloat16* er = p.embed + (size_t)p.tok[r] * d;
-      for (int k0 = 0; k0 * 256 < nc; k0 += NORM_NB) {
-        float4 v[2][NORM_NB];
+      for (int k0 = 0; k0 * CT < nc; k0 += NORM_NB) {
+        float4 v[NORM_NB];
 #pragma unroll
-        for (int s = 0; s < 2; ++s) {
-#pragma unroll
-          for (int k = 0; k < NORM_NB; ++k) {
-            const int c = ctid + 128 * s + 256 * (k0 + k);
-            if (c < nc) {
-              const uint2 raw = *reinterpret_cast<const uint2*>(er + 4 * c);
-              const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&raw);
-              const float2 f0 = __bfloat1622float2(b[0]), f1 = __bfloat1622float2(b[1]);
-              v[s][k] = make_float4(f0.x, f0.y, f1.x, f1.y);
-            }
+        for (int k = 0; k < NORM_NB; ++k) {
+          const int c = ctid + CT * (k0 + k);
+          if (c < nc) {
+            const uint2 raw = *reinterpret_cast<const uint2*>(er + 4 * c);
+            const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&raw);
+            const float2 f0 = __bfloat1622float2(b[0]), f1 = __bfloat1622float2(b[1]);
+            v[k] = make_float4(f0.x, f0.y, f1.x, f1.y);
           }
         }
 #pragma unroll
-        for (int s = 0; s < 2; ++s) {
-#pragma unroll
-          for (int k = 0; k < NORM_NB; ++k) {
-            const int c = ctid + 128 * s + 256 * (k0 + k);
-            if (c < nc) {
-              *reinterpret_cast<float4*>(hr + 4 * c) = v[s][k];
-              rowbuf[c] = v[s][k];
-              ss[s] += v[s][k].x * v[s][k].x;
-              ss[s] += v[s][k].y * v[s][k].y;
-              ss[s] += v[s][k].z * v[s][k].z;
-              ss[s] += v[s][k].w * v[s][k].w;
-            }
+        for (int k = 0; k < NORM_NB; ++k) {
+          const int c = ctid + CT * (k0 + k);
+          if (c < nc) {
+            *reinterpret_cast<float4*>(hr + 4 * c) = v[k];
+            rowbuf[c] = v[k];
+            ss += v[k].x * v[k].x;
+            ss += v[k].y * v[k].y;
+            ss += v[k].z * v[k].z;
+            ss += v[k].w * v[k].w;
           }
         }
       }
@@ -358,18 +355,18 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
         build_part_table<BN>(p, gi_prev, nt, toff, tslot, ctid);
         tab_nt = gi_prev * 65536 + nt;
       }
-      // h += product: warp w takes m-tiles w, w + 4, ...; a lane four rows of each
+      // h += product: warp w takes m-tiles w, w + 8, ...; a lane four rows of each
       const int mtn = (d + GEMM_BM - 1) / GEMM_BM;
       const float4* ws4 = reinterpret_cast<const float4*>(p.ws);
       constexpr long long SLOT4 = GEMM_WS_SLOT_FLOATS / 4;
       const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
       for (int t0 = w; t0 < mtn; t0 += 32) {
-        float4 acc[8], hv[8];
-        int P[8], o[8];
+        float4 acc[4], hv[4];
+        int P[4], o[4];
         int Pm = 0;
 #pragma unroll
-        for (int b = 0; b < 8; ++b) {
-          const int mt = t0 + 4 * b;
+        for (int b = 0; b < 4; ++b) {
+          const int mt = t0 + 8 * b;
           const bool in = mt < mtn && mt * GEMM_BM + 4 * lane < d;
           P[b] = in ? toff[mt + 1] - toff[mt] : 0;
           o[b] = in ? toff[mt] : 0;
@@ -380,12 +377,12 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
         }
 #pragma unroll 2
         for (int e = 0; e < Pm; ++e) {
-          float4 v[8];
+          float4 v[4];
 #pragma unroll
-          for (int b = 0; b < 8; ++b)
+          for (int b = 0; b < 4; ++b)
             if (e < P[b]) v[b] = __ldcg(ws4 + (long long)tslot[o[b] + e] * SLOT4 + j * (GEMM_BM / 4) + lane);
 #pragma unroll
-          for (int b = 0; b < 8; ++b) {
+          for (int b = 0; b < 4; ++b) {
             if (e < P[b]) {
               acc[b].x += v[b].x;
               acc[b].y += v[b].y;
@@ -395,8 +392,8 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
           }
         }
 #pragma unroll
-        for (int b = 0; b < 8; ++b) {
-          const int mt = t0 + 4 * b;
+        for (int b = 0; b < 4; ++b) {
+          const int mt = t0 + 8 * b;
           if (mt < mtn && mt * GEMM_BM + 4 * lane < d) {
             const float4 v = make_float4(hv[b].x + acc[b].x, hv[b].y + acc[b].y, hv[b].z + acc[b].z,
                                          hv[b].w + acc[b].w);
@@ -405,32 +402,24 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
           }
         }
       }
-      named_bar_sync(1, 128);
+      named_bar_sync(1, CT);
       if (p.trace && ctid == 0 && r == (int)blockIdx.x) p.trace[((size_t)4 * (7 * p.L + 2) + ph) * p.G + blockIdx.x] = globaltimer_ns();
-#pragma unroll
-      for (int s = 0; s < 2; ++s) {
-        for (int k = 0;; ++k) {
-          const int c = ctid + 128 * s + 256 * k;
-          if (c >= nc) break;
-          const float4 v = rowbuf[c];
-          ss[s] += v.x * v.x;
-          ss[s] += v.y * v.y;
-          ss[s] += v.z * v.z;
-          ss[s] += v.w * v.w;
-        }
+      for (int c = ctid; c < nc; c += CT) {
+        const float4 v = rowbuf[c];
+        ss += v.x * v.x;
+        ss += v.y * v.y;
+        ss += v.z * v.z;
+        ss += v.w * v.w;
       }
     }
-    const float sa = warp_sum(ss[0]), sb = warp_sum(ss[1]);
-    if (lane == 0) {
-      red[w] = sa;
-      red[w + 4] = sb;
-    }
-    named_bar_sync(1, 128);
+    ss = warp_sum(ss);
+    if (lane == 0) red[w] = ss;
+    named_bar_sync(1, CT);
     if (p.trace && ctid == 0 && r == (int)blockIdx.x) p.trace[((size_t)5 * (7 * p.L + 2) + ph) * p.G + blockIdx.x] = globaltimer_ns();
     const float rs = 1.0f / sqrtf(rms_total(red) / (float)d + p.eps);
     __nv_bfloat16* xr = p.x + (size_t)r * d;
 #pragma unroll 4
-    for (int c = ctid; c < nc; c += 128) {
+    for (int c = ctid; c < nc; c += CT) {
       const float4 v = rowbuf[c];
       const uint2 graw = *reinterpret_cast<const uint2*>(g + 4 * c);
       const __nv_bfloat162* gb = reinterpret_cast<const __nv_bfloat162*>(&graw);
@@ -440,15 +429,16 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
       o[1] = __floats2bfloat162_rn(v.z * rs * g1.x, v.w * rs * g1.y);
       *reinterpret_cast<uint2*>(xr + 4 * c) = *reinterpret_cast<uint2*>(o);
     }
-    named_bar_sync(1, 128);
+    named_bar_sync(1, CT);
   }
 }
 
-// Tree attention of layer l: this CTA's work items (query tile, head, prefix split), each followed
-// by its share of the merge of the splits of (tile, head).
+// Tree attention of layer l, one warpgroup (128 threads, `wt`): its work items (query tile, head,
+// prefix split) are item c + (2k + wg) G; each is followed by the warpgroup's share of the merge of
+// the splits of (tile, head) once all of them are published.
 template <int HD>
 __device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* att_smem, uint64_t* att_bars, int* s_info,
-                                        int (&use_att)[2], int* flag, int ctid) {
+                                           int (&use_att)[2], int* flag, int wt, int wg, int wbar) {
   const int c = blockIdx.x, G = p.G, L = p.L;
   AttnArgs a = p.att_args;
   a.k_cache = p.kc + p.layer_elems * l;
@@ -458,62 +448,73 @@ __device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* a
   const int H = p.H, S = a.max_splits;
   const int NP = 7 * L + 2, ph = 7 * l + 2;
   int nit = 0;
-  for (int item = c; item < p.att_items; item += G, ++nit) {
+  for (int item = c + wg * G; item < p.att_items; item += 2 * G, ++nit) {
     const int tile = item / (H * S), rem = item % (H * S);
     const int h = rem / S, split = rem % S;
-    unsigned long long* tr = (p.trace && nit == 0) ? p.trace + ((size_t)8 * NP + ph) * G + c : nullptr;
-    if (!attn_item<HD>(a, mk, mv, tile, h, split, att_smem, att_bars, s_info, use_att, ctid, 1, tr, (size_t)NP * G))
+    const bool tr_on = p.trace && wg == 0 && nit == 0;
+    unsigned long long* tr = tr_on ? p.trace + ((size_t)8 * NP + ph) * G + c : nullptr;
+    if (!attn_item<HD>(a, mk, mv, tile, h, split, att_smem, att_bars, s_info, use_att, wt, wbar, tr, (size_t)NP * G))
       return false;
-    if (p.trace && ctid == 0 && nit < 2) p.trace[((size_t)(4 + 2 * nit) * NP + ph) * G + c] = globaltimer_ns();
+    if (tr_on && wt == 0) p.trace[((size_t)4 * NP + ph) * G + c] = globaltimer_ns();
     if (a.direct) continue;
     const int S_u = a.user_splits[a.qt_user[tile]];
     if (split >= S_u) continue;
-    // every split publishes its partials and waits for the others of (tile, h) -- they run in the
-    // same or a later round of items, never an earlier one -- then split s merges query groups
-    // s, s + S_u, ...  The counter only grows during a launch: layer l completes at S_u * (l + 1).
+    // every split publishes its partials and waits for the others of (tile, h) -- all items run in
+    // one round (2 G work slots), or the awaited ones in a later round, never an earlier one -- then
+    // split s merges query groups s, s + S_u, ...  The counter only grows during a launch: layer l
+    // completes at S_u * (l + 1).
     __threadfence();
-    named_bar_sync(1, 128);
-    if (ctid == 0) {
+    named_bar_sync(wbar, 128);
+    if (wt == 0) {
       int* cnt = &p.att_counters[tile * H + h];
       atomicAdd(cnt, 1);
       *flag = counter_wait(cnt, S_u * (l + 1), p.err) ? 1 : 0;
     }
-    named_bar_sync(1, 128);
+    named_bar_sync(wbar, 128);
     if (!*flag) return false;
     const int nq = a.qt_n[tile];
-    for (int qg = split; qg * ATT_CQ < nq; qg += S_u) attn_combine_group<HD>(a, tile, h, qg, ctid);
-    named_bar_sync(1, 128);
-    if (p.trace && ctid == 0 && nit < 2) p.trace[((size_t)(5 + 2 * nit) * NP + ph) * G + c] = globaltimer_ns();
+    for (int qg = split; qg * ATT_CQ < nq; qg += S_u) attn_combine_group<HD>(a, tile, h, qg, wt);
+    named_bar_sync(wbar, 128);
+    if (tr_on && wt == 0) p.trace[((size_t)5 * NP + ph) * G + c] = globaltimer_ns();
   }
   return true;
 }
 
-// GEMM phase gi (program phase ph), compute-warp side.  For each of this CTA's segments, wait for
-// its accumulator, then:
+// GEMM phase gi (program phase ph), compute-warp side (256 threads, ctid).  The 32-token chunks of
+// a tile alternate between the two warpgroups (chunk ch by warpgroup ch & 1, each with its own
+// staging buffer and named barrier); warp 4 + q and warp 8 + q both read TMEM lane quadrant q.
+// For each of this CTA's segments, wait for its accumulator, then:
 //  * O / down projections (to_dh): a whole tile goes to dh, a split tile's part to this CTA's
-//    workspace slot ([token][row] layout); the next norm phase sums the parts (no reduction here);
+//    workspace slot ([token][row] layout); the next norm phase sums the parts;
 //  * other GEMMs: a whole tile runs the fused epilogue; for a split tile, if every other part is
-//    already published this CTA is the last one and sums the parts with its own part read straight
-//    from TMEM; otherwise it publishes its part and the last CTA to arrive does the sum.
+//    already published (and this is the CTA's last segment) this CTA is the last one and sums the
+//    parts with its own part read straight from TMEM; otherwise it publishes its part and the last
+//    CTA to arrive does the sum.
+//  * shared sums (phases with whole tiles per CTA, whose split tiles come first and finish early,
+//    and the LM head, whose tiles have many short parts): every part publishes, then each part sums
+//    a share of its tile's chunks (chunk ch by part ch mod parts).
 // Parts are always summed in k order starting from zero, whichever CTA sums them.  Kept out of
 // line so that the epilogue gets its own register allocation.
 template <int BN>
-__device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, float* staging, uint64_t* tfull,
+__device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, float* staging_base, uint64_t* tfull,
                                             uint64_t* tempty, int* flag, int* part_slot, int* tpos, int* tkvr,
                                             uint32_t tmem_base, int ctid, int& si) {
   const int c = blockIdx.x, G = p.G, NP = 7 * p.L + 2;
-  const int lane = ctid & 31, q = ctid >> 5, m = ctid;   // warp 4 + q reads TMEM lane quadrant q
+  const int wg = ctid >> 7, wt = ctid & 127, wbar = 2 + wg;
+  const int lane = ctid & 31, q = (ctid >> 5) & 3, m = wt;   // TMEM lane quadrant q, row m of the tile
+  float* staging = staging_base + wg * (32 * GEMM_BM);
   const GP g = gemm_phase(p, gi, BN);
   const GemmArgs ea = epi_args(p, g);
   const int kb = g.kb;
   SegIter it;
   it.init(g.w, c);
   int tile, k0, k1;
-  // Shared sums: in a phase with whole tiles per CTA the split (stream-K) tiles come first and
-  // finish early; in the LM head every tile is split into many short parts (and no CTA has more
-  // than two segments).  Every part publishes its partial sum (all of this CTA's, before any wait),
-  // then each part sums a share of its tile's chunks (chunk ch by part ch mod parts) -- spread over
-  // the parts' CTAs instead of one.
+  auto fill_part_slots = [&](long long tu0, int c_first, int parts) {
+    for (int pi = ctid; pi < parts; pi += CT) {
+      const int cc = c_first + pi;
+      part_slot[pi] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
+    }
+  };
   const bool shared_sums = !g.to_dh && (g.w.q > 0 || (gi == 4 * p.L && g.w.Gsk > 0 && g.w.Usk / g.w.Gsk + 1 < kb));
   if (shared_sums && it.u < it.u1) {
     int sk_tile[2], nsk = 0;
@@ -521,19 +522,18 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       it.next(g.w, tile, k0, k1);
       const int acc = si & 1, use = si >> 1;
       ++si;
-      const bool got = mwait(&tfull[acc], (uint32_t)(use & 1), p.err);
-      __syncwarp();
+      const bool got = named_bar_and(1, CT, mwait(&tfull[acc], (uint32_t)(use & 1), p.err));
       if (!got) return false;
       tc_fence_after();
       const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       const int nch = min(BN / 32, (g.rows - (tile % g.n_tiles) * BN + 31) / 32);
-      ws_store_partial(p.ws + ((long long)c * 2 + nsk) * GEMM_WS_SLOT_FLOATS, tb, nch, m);
+      ws_store_partial(p.ws + ((long long)c * 2 + nsk) * GEMM_WS_SLOT_FLOATS, tb, nch, m, wg, 2);
       tc_fence_before();
       if (lane == 0) mbar_arrive(&tempty[acc]);
       sk_tile[nsk++] = tile;
     }
     __threadfence();
-    named_bar_sync(1, 128);
+    named_bar_sync(1, CT);
     int* skc = p.sk_counters + (size_t)gi * G;
     if (ctid == 0)
       for (int j = 0; j < nsk; ++j) atomicAdd(&skc[sk_tile[j]], 1);
@@ -543,42 +543,41 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       const int c_first = sk_owner(g.w, tu0);
       const int parts = sk_owner(g.w, tu0 + kb - 1) - c_first + 1;
       const int m_tile = t / g.n_tiles, n_tile = t % g.n_tiles;
-      for (int pi = ctid; pi < parts; pi += 128) {
-        const int cc = c_first + pi;
-        part_slot[pi] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
-      }
-      if (g.epi == EPI_QKV) load_tok_tables<BN>(ea, n_tile, tpos, tkvr, ctid);
+      fill_part_slots(tu0, c_first, parts);
+      if (g.epi == EPI_QKV) load_tok_tables<BN>(ea, n_tile, tpos, tkvr, ctid, CT);
       if (ctid == 0) *flag = counter_wait(&skc[t], parts, p.err) ? 1 : 0;
-      named_bar_sync(1, 128);
+      named_bar_sync(1, CT);
       if (!*flag) return false;
       const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
-      for (int ch = c - c_first; ch < nch; ch += parts) {
-        ws_reduce_chunk(p.ws, part_slot, parts, ch, m, staging);
-        named_bar_sync(1, 128);
-        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid, tpos, tkvr);
-        named_bar_sync(1, 128);
+      int k = 0;
+      for (int ch = c - c_first; ch < nch; ch += parts, ++k) {
+        if ((k & 1) != wg) continue;
+        ws_reduce_chunk<2>(p.ws, part_slot, parts, ch, m, staging);
+        named_bar_sync(wbar, 128);
+        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        named_bar_sync(wbar, 128);
       }
-      named_bar_sync(1, 128);   // flag, part_slot and the token tables are reused
+      named_bar_sync(1, CT);   // flag, part_slot and the token tables are reused
     }
   }
   for (int seg = 0; it.next(g.w, tile, k0, k1); ++si, ++seg) {
     const int acc = si & 1, use = si >> 1;
     const int m_tile = tile / g.n_tiles, n_tile = tile % g.n_tiles;
     const bool whole = (k0 == 0 && k1 == kb);
-    if (g.epi == EPI_QKV) load_tok_tables<BN>(ea, n_tile, tpos, tkvr, ctid);
+    if (g.epi == EPI_QKV) {
+      named_bar_sync(1, CT);   // both warpgroups are done with the previous segment's token tables
+      load_tok_tables<BN>(ea, n_tile, tpos, tkvr, ctid, CT);
+    }
     long long tu0 = 0;
     int c_first = 0, parts = 1;
     if (!whole && !g.to_dh) {
       tu0 = (long long)tile * kb;
       c_first = sk_owner(g.w, tu0);
       parts = sk_owner(g.w, tu0 + kb - 1) - c_first + 1;
-      for (int pi = ctid; pi < parts; pi += 128) {
-        const int cc = c_first + pi;
-        part_slot[pi] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
-      }
+      fill_part_slots(tu0, c_first, parts);
     }
-    const bool got = mwait(&tfull[acc], (uint32_t)(use & 1), p.err);
-    __syncwarp();
+    // (the vote is also the barrier after which token tables and part slots are in place)
+    const bool got = named_bar_and(1, CT, mwait(&tfull[acc], (uint32_t)(use & 1), p.err));
     if (!got) return false;
     tc_fence_after();
     if (p.trace && ctid == 0) p.trace[((size_t)4 * NP + ph) * G + c] = globaltimer_ns();
@@ -595,7 +594,7 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
         dst = p.ws + ((long long)c * 2 + (seg == 0 ? 0 : 1)) * GEMM_WS_SLOT_FLOATS + m;
         ld = GEMM_BM;
       }
-      for (int ch = 0; ch < nch; ++ch) {
+      for (int ch = wg; ch < nch; ch += 2) {
         uint32_t r[32];
         tmem_ld_32x32b_x32(tb + ch * 32, r);
         tmem_ld_wait();
@@ -611,15 +610,15 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       continue;
     }
     if (whole) {
-      for (int ch = 0; ch < nch; ++ch) {
+      for (int ch = wg; ch < nch; ch += 2) {
         uint32_t r[32];
         tmem_ld_32x32b_x32(tb + ch * 32, r);
         tmem_ld_wait();
 #pragma unroll
         for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = __uint_as_float(r[j]);
-        named_bar_sync(1, 128);
-        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid, tpos, tkvr);
-        named_bar_sync(1, 128);
+        named_bar_sync(wbar, 128);
+        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        named_bar_sync(wbar, 128);
       }
       tc_fence_before();
       if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -630,33 +629,32 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
     if (ctid == 0)
       *flag = !it.more() &&
               (int)ld_acquire_u32(reinterpret_cast<const unsigned*>(&p.counters[tile])) == parts - 1;
-    named_bar_sync(1, 128);
+    named_bar_sync(1, CT);
     if (*flag) {
       // last part: nobody else touches this tile's counter in this phase
       if (ctid == 0) p.counters[tile] = 0;
       if (p.trace && ctid == 0) p.trace[((size_t)6 * NP + ph) * G + c] = globaltimer_ns();
       const int own = c - c_first;
-      for (int ch = 0; ch < nch; ++ch) {
+      for (int ch = wg; ch < nch; ch += 2) {
         uint32_t r[32];
         tmem_ld_32x32b_x32(tb + ch * 32, r);
         tmem_ld_wait();
         ws_reduce_chunk_own(p.ws, part_slot, parts, own, r, ch, m, staging);
-        named_bar_sync(1, 128);
-        if (p.trace && ctid == 0 && ch < 4) p.trace[((size_t)(8 + 2 * ch) * NP + ph) * G + c] = globaltimer_ns();
-        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid, tpos, tkvr);
-        named_bar_sync(1, 128);
-        if (p.trace && ctid == 0 && ch < 4) p.trace[((size_t)(9 + 2 * ch) * NP + ph) * G + c] = globaltimer_ns();
+        named_bar_sync(wbar, 128);
+        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        named_bar_sync(wbar, 128);
       }
       tc_fence_before();
       if (lane == 0) mbar_arrive(&tempty[acc]);
+      named_bar_sync(1, CT);   // flag and part_slot are reused by the next segment
       continue;
     }
     const long long slot = (long long)c * 2 + (seg == 0 ? 0 : 1);
-    ws_store_partial(p.ws + slot * GEMM_WS_SLOT_FLOATS, tb, nch, m);
+    ws_store_partial(p.ws + slot * GEMM_WS_SLOT_FLOATS, tb, nch, m, wg, 2);
     tc_fence_before();
     if (lane == 0) mbar_arrive(&tempty[acc]);
     __threadfence();
-    named_bar_sync(1, 128);
+    named_bar_sync(1, CT);
     if (p.trace && ctid == 0) p.trace[((size_t)5 * NP + ph) * G + c] = globaltimer_ns();
     if (ctid == 0) {
       const int old = atomicAdd(&p.counters[tile], 1);
@@ -667,19 +665,17 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       }
       *flag = last;
     }
-    named_bar_sync(1, 128);
+    named_bar_sync(1, CT);
     if (p.trace && ctid == 0) p.trace[((size_t)6 * NP + ph) * G + c] = globaltimer_ns();
     if (*flag) {
-      for (int ch = 0; ch < nch; ++ch) {
-        ws_reduce_chunk(p.ws, part_slot, parts, ch, m, staging);
-        named_bar_sync(1, 128);
-        if (p.trace && ctid == 0 && ch < 4) p.trace[((size_t)(8 + 2 * ch) * NP + ph) * G + c] = globaltimer_ns();
-        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, ctid, tpos, tkvr);
-        named_bar_sync(1, 128);
-        if (p.trace && ctid == 0 && ch < 4) p.trace[((size_t)(9 + 2 * ch) * NP + ph) * G + c] = globaltimer_ns();
+      for (int ch = wg; ch < nch; ch += 2) {
+        ws_reduce_chunk<2>(p.ws, part_slot, parts, ch, m, staging);
+        named_bar_sync(wbar, 128);
+        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        named_bar_sync(wbar, 128);
       }
     }
-    named_bar_sync(1, 128);  // flag and part_slot are reused by the next segment
+    named_bar_sync(1, CT);  // flag and part_slot are reused by the next segment
   }
   return true;
 }
@@ -702,21 +698,22 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
   uint64_t* tfull = emptyB + C::SB;
   uint64_t* tempty = tfull + 2;
   uint64_t* mma_done = tempty + 2;
-  uint64_t* att_bars = mma_done + 1;                              // 2
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(att_bars + 2);
+  uint64_t* att_bars = mma_done + 1;                              // 2 per warpgroup
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(att_bars + 4);
   int* flag = reinterpret_cast<int*>(tmem_slot + 1);
-  int* failed = flag + 1;
+  int* flagw = flag + 1;                                          // 2: one per warpgroup
+  int* failed = flagw + 2;
   int* go = failed + 1;   // count of GEMM phases whose input the compute warps have seen published
   int* lastA = go + 1;                                            // [SA] parity of last fill, -1 none
   int* lastB = lastA + C::SA;                                     // [SB]
-  int* s_info = lastB + C::SB;                                    // 6 (attention)
-  float* red = reinterpret_cast<float*>(s_info + 6);              // 8
+  int* s_info = lastB + C::SB;                                    // 6 per warpgroup (attention)
+  float* red = reinterpret_cast<float*>(s_info + 12);             // 8
   int* part_slot = reinterpret_cast<int*>(red + 8);               // 256
   int* tpos = part_slot + 256;                                    // [BN] QKV token tables
   int* tkvr = tpos + 256;
   int* toff = tkvr + 256;                                         // [65] part table (norm phases)
   int* tslot = toff + 68;                                         // [PART_TABLE_CAP]
-  static_assert(8 * (2 * C::SA + 2 * C::SB + 7) + 4 * (4 + C::SA + C::SB + 6 + 8 + 256 + 512 + 68 + PART_TABLE_CAP) <=
+  static_assert(8 * (2 * C::SA + 2 * C::SB + 9) + 4 * (6 + C::SA + C::SB + 12 + 8 + 256 + 512 + 68 + PART_TABLE_CAP) <=
                     C::MISC,
                 "shared-memory misc area too small");
 
@@ -738,9 +735,9 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], 4);
-      mbar_init(&att_bars[i], 1);
+      mbar_init(&tempty[i], 8);   // one arrival per compute warp
     }
+    for (int i = 0; i < 4; ++i) mbar_init(&att_bars[i], 1);
     mbar_init(mma_done, 1);
     *go = 0;
     *failed = 0;
@@ -884,10 +881,9 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
       mbar_wait(mma_done, (uint32_t)(mma_waits & 1), nullptr);
     }
   } else if (warp >= COMPUTE_WARP0) {
-    // ------------------------------------------------------------- compute warps
+    // ------------------------------------------------------------- compute warps (two warpgroups)
     const int ctid = threadIdx.x - COMPUTE_WARP0 * 32;
-    const int q = warp & 3;      // TMEM lane quadrant
-    const int m = q * 32 + lane;
+    const int wg = ctid >> 7, wt = ctid & 127;
     int si = 0;
     int use_att[2] = {0, 0};
     int tab_nt = -1;   // (GEMM phase, n-tile) whose part table is in toff / tslot
@@ -936,13 +932,13 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
           *flag = grid_wait(p, ph - 1) ? 1 : 0;
           if (*flag && kind == 1) st_release_cta(go, gi + 1);
         }
-        named_bar_sync(1, 128);
+        named_bar_sync(1, CT);
         if (!*flag) {
           ok = false;
           break;
         }
         fence_proxy_async();
-        named_bar_sync(1, 128);
+        named_bar_sync(1, CT);
       }
       if (kind == 0 || kind == 3 || kind == 4) {
         const int nmode = kind == 0 ? 0 : (kind == 4 && l + 1 == L) ? 2 : 1;
@@ -950,7 +946,10 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
                                   : (l + 1 < L ? p.attn_norm[l + 1] : p.final_norm);
         norm_phase<BN>(p, nmode, ng, red, rowbuf, ctid, 4 * l + (kind == 3 ? 1 : 3), toff, tslot, tab_nt, ph);
       } else if (kind == 2) {
-        if (!attn_phase<HD>(p, l, att_smem, att_bars, s_info, use_att, flag, ctid)) {
+        // both warpgroups leave together: a failed bounded wait in either ends the program
+        const bool aok = attn_phase<HD>(p, l, att_smem + wg * LY::ATT_BODY, att_bars + 2 * wg, s_info + 6 * wg,
+                                        use_att, flagw + wg, wt, wg, 2 + wg);
+        if (!named_bar_and(1, CT, aok)) {
           ok = false;
           break;
         }
@@ -966,7 +965,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
       if (ph < NP - 1) {
         fence_proxy_async();
         __threadfence();
-        named_bar_sync(1, 128);
+        named_bar_sync(1, CT);
         if (ctid == 0) atomicAdd(p.bar, 1u);
       }
     }

@@ -225,8 +225,7 @@ __global__ void __launch_bounds__(192, 1)
     int tile, k0, k1;
     for (; it.next(p.w, tile, k0, k1); ++si) {
       const int acc = si & 1, use = si >> 1;
-      const bool got = mbar_wait(&tfull[acc], (uint32_t)(use & 1), p.err);
-      __syncwarp();
+      const bool got = named_bar_and(1, 128, mbar_wait(&tfull[acc], (uint32_t)(use & 1), p.err));
       if (!got) {
         *failed = 1;
         break;

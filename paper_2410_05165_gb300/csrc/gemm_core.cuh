@@ -97,8 +97,9 @@ struct SegIter {
 // row), copied to shared memory when a segment starts so that the epilogue's loads do not wait on
 // them.  Callers synchronise the 128 threads before the first chunk's epilogue.
 template <int BN>
-__device__ __forceinline__ void load_tok_tables(const GemmArgs& a, int n_tile, int* tpos, int* tkvr, int ep_tid) {
-  for (int j = ep_tid; j < BN; j += 128) {
+__device__ __forceinline__ void load_tok_tables(const GemmArgs& a, int n_tile, int* tpos, int* tkvr, int ep_tid,
+                                                int nthreads = 128) {
+  for (int j = ep_tid; j < BN; j += nthreads) {
     const int tok = n_tile * BN + j;
     tpos[j] = tok < a.T ? a.pos[tok] : 0;
     tkvr[j] = tok < a.T ? a.kv_row[tok] : 0;
@@ -200,10 +201,10 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, in
 // A workspace slot holds one CTA's fp32 partial of a 128-row tile for up to 256 tokens, laid out
 // [token/4][row][4] so that a thread (one weight row) moves four tokens per 16-byte access.
 
-// TMEM accumulator (this thread's lane = row m) -> workspace slot, chunks [0, nch)
-__device__ __forceinline__ void ws_store_partial(float* wsl, uint32_t tb, int nch, int m) {
+// TMEM accumulator (this thread's lane = row m) -> workspace slot, chunks ch0, ch0 + step, ... < nch
+__device__ __forceinline__ void ws_store_partial(float* wsl, uint32_t tb, int nch, int m, int ch0 = 0, int step = 1) {
   float4* w4 = reinterpret_cast<float4*>(wsl);
-  for (int ch = 0; ch < nch; ++ch) {
+  for (int ch = ch0; ch < nch; ch += step) {
     uint32_t r[32];
     tmem_ld_32x32b_x32(tb + ch * 32, r);
     tmem_ld_wait();
@@ -216,7 +217,9 @@ __device__ __forceinline__ void ws_store_partial(float* wsl, uint32_t tb, int nc
 }
 
 // Sum, in k order (part 0 first, starting from zero), of chunk ch of the parts in `slot` -> this
-// thread's row m of the staging buffer [32 tokens][128 rows].  Up to four parts are in flight at once.
+// thread's row m of the staging buffer [32 tokens][128 rows].  PB parts are in flight at once (the
+// result does not depend on PB).
+template <int PB = 4>
 __device__ __forceinline__ void ws_reduce_chunk(const float* ws, const int* slot, int parts, int ch, int m,
                                                 float* staging) {
   float acc[32];
@@ -224,10 +227,10 @@ __device__ __forceinline__ void ws_reduce_chunk(const float* ws, const int* slot
   for (int j = 0; j < 32; ++j) acc[j] = 0.f;
   const float4* w4 = reinterpret_cast<const float4*>(ws);
   constexpr long long SLOT4 = GEMM_WS_SLOT_FLOATS / 4;
-  for (int p0 = 0; p0 < parts; p0 += 4) {
-    float4 v[4][8];
+  for (int p0 = 0; p0 < parts; p0 += PB) {
+    float4 v[PB][8];
 #pragma unroll
-    for (int b = 0; b < 4; ++b) {
+    for (int b = 0; b < PB; ++b) {
       if (p0 + b < parts) {
         const float4* src = w4 + (long long)slot[p0 + b] * SLOT4 + (ch * 8) * GEMM_BM + m;
 #pragma unroll
@@ -235,7 +238,7 @@ __device__ __forceinline__ void ws_reduce_chunk(const float* ws, const int* slot
       }
     }
 #pragma unroll
-    for (int b = 0; b < 4; ++b) {
+    for (int b = 0; b < PB; ++b) {
       if (p0 + b < parts) {
 #pragma unroll
         for (int j4 = 0; j4 < 8; ++j4) {
