@@ -29,7 +29,7 @@ namespace {
 
 thread_local std::string g_create_error;
 
-constexpr int kChunksPerSplit = 4;  // prefix pages per attention split (tree queries)
+constexpr int kChunksPerSplit = 2;  // prefix pages per attention split (tree queries)
 
 struct Fail {
   atspeed_status st;
