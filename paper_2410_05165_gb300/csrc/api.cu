@@ -37,6 +37,7 @@ struct Fail {
 
 struct ModelRt {
   bool present = false;
+  bool per_op = false;   // this model's forward runs one kernel per op (else one persistent launch)
   int layers = 0, d = 0, H = 0, hd = 0, ffn = 0, V = 0;
   float eps = 1e-6f, theta = 1e4f;
   const bf16 *embed = nullptr, *final_norm = nullptr, *lm_head = nullptr;
@@ -135,7 +136,7 @@ struct atspeed_ctx {
   std::vector<ProfRec> prof_recs;
   std::vector<cudaEvent_t> prof_pool;
   long long n_launch = 0;  // kernels launched by this context (all kinds)
-  bool per_op = false;     // one kernel per op instead of the persistent single-launch forward
+  int forward_mode = 0;    // ATSPEED_FORWARD: 0 by model size, 1 persistent, 2 one kernel per op
   int fwd_grid = 0;
   unsigned int* fwd_bar = nullptr;
   int* fwd_sk = nullptr;     // split-tile arrival counters of the persistent forward
@@ -521,7 +522,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
   for (int s : p.splits) max_split = std::max(max_split, s);
   const size_t per = (size_t)m.rows * m.d;
   const bool pdl = c->pdl;
-  if (!c->per_op) {
+  if (!m.per_op) {
     // the whole forward in one persistent cooperative launch
     if (nqt > m.max_qt) {
       set_err(c, "forward needs %d query tiles (capacity %d)", nqt, m.max_qt);
@@ -1208,9 +1209,16 @@ atspeed_status atspeed_create(const atspeed_model_desc* target, const atspeed_mo
     c->gemm_grid = gemm_grid_size(c->device);
     c->fwd_grid = c->gemm_grid;  // one persistent CTA per SM
     {
-      // the forward runs as one persistent launch; ATSPEED_FORWARD=per_op selects one kernel per op
+      // Schedule of a model's forward: one persistent launch for models whose layer weights reach
+      // 1 GB (the weight stream then dwarfs the phase latencies), one kernel per op below that (a
+      // few-layer draft model, where the per-op kernels' shorter phases win).  ATSPEED_FORWARD=
+      // persistent | per_op forces one schedule for both models.
       const char* fm = getenv("ATSPEED_FORWARD");
-      c->per_op = fm && strcmp(fm, "per_op") == 0;
+      c->forward_mode = (fm && strcmp(fm, "persistent") == 0) ? 1 : (fm && strcmp(fm, "per_op") == 0) ? 2 : 0;
+      for (ModelRt* mr : {&c->tgt, &c->drf}) {
+        const double wbytes = 2.0 * mr->layers * (4.0 * mr->d * mr->d + 3.0 * mr->d * mr->ffn);
+        mr->per_op = c->forward_mode == 2 || (c->forward_mode == 0 && wbytes < 1e9);
+      }
     }
     c->fwd_bar = dalloc<unsigned int>(c, 1);
     {
