@@ -278,3 +278,36 @@ def test_persistent_forward_equals_per_op_kernels(ats, cfg, layers, monkeypatch)
         ctx.close()
     np.testing.assert_array_equal(outs[0][0], outs[1][0])
     np.testing.assert_array_equal(outs[0][1], outs[1][1])
+
+
+@pytest.mark.parametrize("cfg,layers,B", [("tiny", None, 5), ("mid", 2, 3)])
+def test_persistent_forward_equals_per_op_multi_user(ats, cfg, layers, B, monkeypatch):
+    """Several users with different prompt lengths in one verification call (their own prefix pages,
+    query tiles and attention splits): the two schedules give the same logits, bit for bit, for
+    every user's prefill row and tree nodes."""
+    w = synth.workload(cfg)
+    spec = w.target if layers is None else synth.ModelSpec(layers, w.target.d_model, w.target.n_heads,
+                                                          w.target.d_ffn, w.target.vocab)
+    items = synth.make_items(min(w.n_items, 5000), w.code_dist, w.zipf_a, w.seed)
+    full = synth.make_prompts(B, w.prompt_len, spec.vocab, w.seed)
+    prompts = [p[: max(1, len(p) - 37 * u)] for u, p in enumerate(full)]   # ragged prefixes
+    K, N, G = w.K, w.N, 3
+    _, levels = synth.random_tree(items, 0, 1, G, N, seed=11)
+    cnt1, par1, cod1, sq1 = _tree_arrays(levels, 1, G, N)
+    cnt, par, cod, sq = (np.repeat(a, B, axis=0) for a in (cnt1, par1, cod1, sq1))
+    outs = []
+    for mode in ("per_op", "persistent"):
+        monkeypatch.setenv("ATSPEED_FORWARD", mode)
+        ctx = _ctx(ats, spec, None, items, w.code_base, B, max(len(p) for p in prompts), K, N, G, seed=w.seed)
+        _prefill(ats, ctx, prompts)
+        o = ats.opts(K, N, G)
+        ctx.begin_step(o)
+        ctx.set_tree(cnt, par, cod, sq)
+        ctx.verify(o, ats.STRICT)
+        got = [np.stack([ctx.node_logits(0, u, 0)] +
+                        [ctx.node_logits(0, u, K + j * N + k) for j, lvl in enumerate(levels) for k in range(len(lvl))])
+               for u in range(B)]
+        outs.append(np.stack(got))
+        ctx.close()
+    assert np.all(np.isfinite(outs[0]))
+    np.testing.assert_array_equal(outs[0], outs[1])
