@@ -11,8 +11,9 @@
 //     and attention;
 //   * the activation ring (B) is filled by a second producer warp that waits for the barrier that
 //     publishes the phase's input.
-// Warp roles (256 threads): 0 weight TMA, 1 activation TMA, 2 TMEM + MMA issue, 3 idle,
-// 4..7 compute (GEMM epilogues on TMEM lane quadrants 0..3, RMSNorm rows, tree attention).
+// Warp roles (384 threads): 0 weight TMA, 1 activation TMA, 2 TMEM + MMA issue, 3 idle; 4..11 two
+// compute warpgroups (GEMM epilogues -- a warp reads the TMEM lane quadrant of its id mod 4 --,
+// RMSNorm rows, tree attention).
 // Every wait is bounded; a timeout (or an error raised by another CTA) makes every role leave its
 // loop, in-flight copies are waited for, TMEM is released.
 #include <cudaTypedefs.h>
@@ -28,7 +29,7 @@ namespace atspeed {
 
 namespace {
 
-constexpr int FWD_THREADS = 384;   // warps 0-3: producers, MMA; warps 4-11: two compute warpgroups
+constexpr int FWD_THREADS = 384;   // warps 0-3: producers, MMA (3 idle); warps 4-11: two compute warpgroups
 constexpr int COMPUTE_WARP0 = 4;
 constexpr int CT = 256;            // compute threads (named barrier 1); warpgroup w uses barrier 2 + w
 constexpr int ITEM_ROWS_FWD = 1024;   // item-code rows of the LM head (4 levels x 256 codes)
@@ -228,12 +229,12 @@ __device__ bool mwait(uint64_t* bar, uint32_t parity, unsigned* err) {
 }
 
 template <int BN>
-__device__ __noinline__ void epi_dispatch(int epi, const GemmArgs& a, const float* st, int mt, int nt, int ch,
+__device__ __noinline__ void epi_dispatch(int epi, const GemmArgs* a, const float* st, int mt, int nt, int ch,
                                              int t, const int* tpos, const int* tkvr) {
   switch (epi) {
-    case EPI_F32: epi_chunk<BN, EPI_F32>(a, st, mt, nt, ch, t, tpos, tkvr); break;
-    case EPI_SWIGLU: epi_chunk<BN, EPI_SWIGLU>(a, st, mt, nt, ch, t, tpos, tkvr); break;
-    default: epi_chunk<BN, EPI_QKV>(a, st, mt, nt, ch, t, tpos, tkvr); break;
+    case EPI_F32: epi_chunk<BN, EPI_F32>(*a, st, mt, nt, ch, t, tpos, tkvr); break;
+    case EPI_SWIGLU: epi_chunk<BN, EPI_SWIGLU>(*a, st, mt, nt, ch, t, tpos, tkvr); break;
+    default: epi_chunk<BN, EPI_QKV>(*a, st, mt, nt, ch, t, tpos, tkvr); break;
   }
 }
 
@@ -498,13 +499,18 @@ __device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* a
 template <int BN>
 __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, float* staging_base, uint64_t* tfull,
                                             uint64_t* tempty, int* flag, int* part_slot, int* tpos, int* tkvr,
-                                            uint32_t tmem_base, int ctid, int& si) {
+                                            GemmArgs* s_ea, uint32_t tmem_base, int ctid, int& si) {
   const int c = blockIdx.x, G = p.G, NP = 7 * p.L + 2;
   const int wg = ctid >> 7, wt = ctid & 127, wbar = 2 + wg;
-  const int lane = ctid & 31, q = (ctid >> 5) & 3, m = wt;   // TMEM lane quadrant q, row m of the tile
+  // a warp reads the TMEM lane quadrant of its warp id mod 4; each warpgroup (4 consecutive warps)
+  // covers all four, so row m of the tile is the quadrant's row of this lane
+  const int lane = ctid & 31, q = (threadIdx.x >> 5) & 3, m = q * 32 + lane;
   float* staging = staging_base + wg * (32 * GEMM_BM);
   const GP g = gemm_phase(p, gi, BN);
-  const GemmArgs ea = epi_args(p, g);
+  // the epilogue's arguments live in shared memory (read by the out-of-line epilogue functions)
+  if (ctid == 0) *s_ea = epi_args(p, g);
+  named_bar_sync(1, CT);
+  const GemmArgs& ea = *s_ea;
   const int kb = g.kb;
   SegIter it;
   it.init(g.w, c);
@@ -552,9 +558,9 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       int k = 0;
       for (int ch = c - c_first; ch < nch; ch += parts, ++k) {
         if ((k & 1) != wg) continue;
-        ws_reduce_chunk<2>(p.ws, part_slot, parts, ch, m, staging);
+        ws_reduce_chunk<1>(p.ws, part_slot, parts, ch, m, staging);
         named_bar_sync(wbar, 128);
-        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
         named_bar_sync(wbar, 128);
       }
       named_bar_sync(1, CT);   // flag, part_slot and the token tables are reused
@@ -617,7 +623,7 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
 #pragma unroll
         for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = __uint_as_float(r[j]);
         named_bar_sync(wbar, 128);
-        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
         named_bar_sync(wbar, 128);
       }
       tc_fence_before();
@@ -641,7 +647,7 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
         tmem_ld_wait();
         ws_reduce_chunk_own(p.ws, part_slot, parts, own, r, ch, m, staging);
         named_bar_sync(wbar, 128);
-        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
         named_bar_sync(wbar, 128);
       }
       tc_fence_before();
@@ -669,9 +675,9 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
     if (p.trace && ctid == 0) p.trace[((size_t)6 * NP + ph) * G + c] = globaltimer_ns();
     if (*flag) {
       for (int ch = wg; ch < nch; ch += 2) {
-        ws_reduce_chunk<2>(p.ws, part_slot, parts, ch, m, staging);
+        ws_reduce_chunk<1>(p.ws, part_slot, parts, ch, m, staging);
         named_bar_sync(wbar, 128);
-        epi_dispatch<BN>(g.epi, ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
         named_bar_sync(wbar, 128);
       }
     }
@@ -713,7 +719,9 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
   int* tkvr = tpos + 256;
   int* toff = tkvr + 256;                                         // [65] part table (norm phases)
   int* tslot = toff + 68;                                         // [PART_TABLE_CAP]
-  static_assert(8 * (2 * C::SA + 2 * C::SB + 9) + 4 * (6 + C::SA + C::SB + 12 + 8 + 256 + 512 + 68 + PART_TABLE_CAP) <=
+  GemmArgs* s_ea = reinterpret_cast<GemmArgs*>((reinterpret_cast<uintptr_t>(tslot + PART_TABLE_CAP) + 15) &
+                                                ~uintptr_t(15));   // epilogue arguments
+  static_assert(8 * (2 * C::SA + 2 * C::SB + 9) + 4 * (6 + C::SA + C::SB + 12 + 8 + 256 + 512 + 68 + PART_TABLE_CAP) + 16 + (int)sizeof(GemmArgs) <=
                     C::MISC,
                 "shared-memory misc area too small");
 
@@ -954,7 +962,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
           break;
         }
       } else {
-        if (!gemm_epi_phase<BN>(p, gi, ph, staging, tfull, tempty, flag, part_slot, tpos, tkvr, tmem_base, ctid, si)) {
+        if (!gemm_epi_phase<BN>(p, gi, ph, staging, tfull, tempty, flag, part_slot, tpos, tkvr, s_ea, tmem_base, ctid, si)) {
           ok = false;
           break;
         }

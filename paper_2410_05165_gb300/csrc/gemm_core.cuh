@@ -221,7 +221,7 @@ __device__ __forceinline__ void ws_store_partial(float* wsl, uint32_t tb, int nc
 // result does not depend on PB).
 template <int PB = 4>
 __device__ __forceinline__ void ws_reduce_chunk(const float* ws, const int* slot, int parts, int ch, int m,
-                                                float* staging) {
+                                             float* staging) {
   float acc[32];
 #pragma unroll
   for (int j = 0; j < 32; ++j) acc[j] = 0.f;
@@ -255,7 +255,7 @@ __device__ __forceinline__ void ws_reduce_chunk(const float* ws, const int* slot
 }
 
 // As ws_reduce_chunk, with part `own` of the sum taken from registers (this CTA's accumulator, 32
-// tokens of row m) instead of the workspace.  Two parts are in flight at once.
+// tokens of row m) instead of the workspace.  One part is in flight at a time.
 __device__ __forceinline__ void ws_reduce_chunk_own(const float* ws, const int* slot, int parts, int own,
                                                     const uint32_t (&r)[32], int ch, int m, float* staging) {
   float acc[32];
@@ -263,30 +263,22 @@ __device__ __forceinline__ void ws_reduce_chunk_own(const float* ws, const int* 
   for (int j = 0; j < 32; ++j) acc[j] = 0.f;
   const float4* w4 = reinterpret_cast<const float4*>(ws);
   constexpr long long SLOT4 = GEMM_WS_SLOT_FLOATS / 4;
-  for (int p0 = 0; p0 < parts; p0 += 2) {
-    float4 v[2][8];
+  for (int pi = 0; pi < parts; ++pi) {
+    if (pi == own) {
 #pragma unroll
-    for (int b = 0; b < 2; ++b) {
-      if (p0 + b < parts && p0 + b != own) {
-        const float4* src = w4 + (long long)slot[p0 + b] * SLOT4 + (ch * 8) * GEMM_BM + m;
-#pragma unroll
-        for (int j4 = 0; j4 < 8; ++j4) v[b][j4] = __ldcg(src + j4 * GEMM_BM);
-      }
+      for (int j = 0; j < 32; ++j) acc[j] += __uint_as_float(r[j]);
+      continue;
     }
+    const float4* src = w4 + (long long)slot[pi] * SLOT4 + (ch * 8) * GEMM_BM + m;
+    float4 v[8];
 #pragma unroll
-    for (int b = 0; b < 2; ++b) {
-      if (p0 + b == own) {
+    for (int j4 = 0; j4 < 8; ++j4) v[j4] = __ldcg(src + j4 * GEMM_BM);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) acc[j] += __uint_as_float(r[j]);
-      } else if (p0 + b < parts) {
-#pragma unroll
-        for (int j4 = 0; j4 < 8; ++j4) {
-          acc[4 * j4] += v[b][j4].x;
-          acc[4 * j4 + 1] += v[b][j4].y;
-          acc[4 * j4 + 2] += v[b][j4].z;
-          acc[4 * j4 + 3] += v[b][j4].w;
-        }
-      }
+    for (int j4 = 0; j4 < 8; ++j4) {
+      acc[4 * j4] += v[j4].x;
+      acc[4 * j4 + 1] += v[j4].y;
+      acc[4 * j4 + 2] += v[j4].z;
+      acc[4 * j4 + 3] += v[j4].w;
     }
   }
 #pragma unroll
