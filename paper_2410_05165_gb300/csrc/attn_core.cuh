@@ -189,78 +189,82 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
     }
     const uint32_t kbase = smem_u32(kvbuf + buf * C::BUF_BYTES);
     const uint32_t vbase = kbase + C::KV_BYTES;
-    float s[8][4];
+    // the page's 64 keys in two halves of 32 (fewer live registers), online softmax over each
+#pragma unroll 1
+    for (int hk = 0; hk < ATT_PAGE / 32; ++hk) {
+      float s[4][4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+      for (int j = 0; j < 4; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
 #pragma unroll
-    for (int jj = 0; jj < 4; ++jj) {
+      for (int jj = 0; jj < 2; ++jj) {
 #pragma unroll
-      for (int kk = 0; kk < NKS; ++kk) {
-        // matrices: (keys 16jj+0..7, dims lo), (keys 0..7, dims hi), (keys 8..15, lo), (keys 8..15, hi)
-        const int key = jj * 16 + (lane & 7) + ((lane >> 4) << 3);
-        const int ch = kk * 2 + ((lane >> 3) & 1);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(kbase + kv_off<HD>(key, ch), b0, b1, b2, b3);
-        mma_bf16_16816(s[2 * jj], qf[kk], b0, b1);
-        mma_bf16_16816(s[2 * jj + 1], qf[kk], b2, b3);
+        for (int kk = 0; kk < NKS; ++kk) {
+          // matrices: (keys 16jj+0..7, dims lo), (keys 0..7, dims hi), (keys 8..15, lo), (keys 8..15, hi)
+          const int key = hk * 32 + jj * 16 + (lane & 7) + ((lane >> 4) << 3);
+          const int ch = kk * 2 + ((lane >> 3) & 1);
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(kbase + kv_off<HD>(key, ch), b0, b1, b2, b3);
+          mma_bf16_16816(s[2 * jj], qf[kk], b0, b1);
+          mma_bf16_16816(s[2 * jj + 1], qf[kk], b2, b3);
+        }
       }
-    }
-    // scale, mask, online softmax (base 2)
-    const int kbase_idx = chunk * ATT_PAGE;
-    float mx_a = m_a, mx_b = m_b;
+      // scale, mask, online softmax (base 2)
+      const int kbase_idx = chunk * ATT_PAGE + hk * 32;
+      float mx_a = m_a, mx_b = m_b;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int k0 = kbase_idx + j * 8 + tq * 2;
-      s[j][0] = (k0 < vis_a) ? s[j][0] * scale : -INFINITY;
-      s[j][1] = (k0 + 1 < vis_a) ? s[j][1] * scale : -INFINITY;
-      s[j][2] = (k0 < vis_b) ? s[j][2] * scale : -INFINITY;
-      s[j][3] = (k0 + 1 < vis_b) ? s[j][3] * scale : -INFINITY;
-      mx_a = fmaxf(mx_a, fmaxf(s[j][0], s[j][1]));
-      mx_b = fmaxf(mx_b, fmaxf(s[j][2], s[j][3]));
-    }
-    mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 1));
-    mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 2));
-    mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 1));
-    mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 2));
-    const float ua = (mx_a == -INFINITY) ? 0.f : mx_a;
-    const float ub = (mx_b == -INFINITY) ? 0.f : mx_b;
-    const float alpha_a = exp2f(m_a - ua), alpha_b = exp2f(m_b - ub);
-    m_a = mx_a;
-    m_b = mx_b;
-    l_a *= alpha_a;
-    l_b *= alpha_b;
+      for (int j = 0; j < 4; ++j) {
+        const int k0 = kbase_idx + j * 8 + tq * 2;
+        s[j][0] = (k0 < vis_a) ? s[j][0] * scale : -INFINITY;
+        s[j][1] = (k0 + 1 < vis_a) ? s[j][1] * scale : -INFINITY;
+        s[j][2] = (k0 < vis_b) ? s[j][2] * scale : -INFINITY;
+        s[j][3] = (k0 + 1 < vis_b) ? s[j][3] * scale : -INFINITY;
+        mx_a = fmaxf(mx_a, fmaxf(s[j][0], s[j][1]));
+        mx_b = fmaxf(mx_b, fmaxf(s[j][2], s[j][3]));
+      }
+      mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 1));
+      mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 2));
+      mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 1));
+      mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 2));
+      const float ua = (mx_a == -INFINITY) ? 0.f : mx_a;
+      const float ub = (mx_b == -INFINITY) ? 0.f : mx_b;
+      const float alpha_a = exp2f(m_a - ua), alpha_b = exp2f(m_b - ub);
+      m_a = mx_a;
+      m_b = mx_b;
+      l_a *= alpha_a;
+      l_b *= alpha_b;
 #pragma unroll
-    for (int j = 0; j < NDT; ++j) {
-      o[j][0] *= alpha_a;
-      o[j][1] *= alpha_a;
-      o[j][2] *= alpha_b;
-      o[j][3] *= alpha_b;
-    }
-    uint32_t ph[4][4];
+      for (int j = 0; j < NDT; ++j) {
+        o[j][0] *= alpha_a;
+        o[j][1] *= alpha_a;
+        o[j][2] *= alpha_b;
+        o[j][3] *= alpha_b;
+      }
+      uint32_t ph[2][4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float p0 = exp2f(s[j][0] - ua), p1 = exp2f(s[j][1] - ua);
-      const float p2 = exp2f(s[j][2] - ub), p3 = exp2f(s[j][3] - ub);
-      l_a += p0 + p1;
-      l_b += p2 + p3;
-      const int kk = j >> 1, r = (j & 1) * 2;
-      const __half2 h01 = __floats2half2_rn(p0, p1), h23 = __floats2half2_rn(p2, p3);
-      ph[kk][r] = *reinterpret_cast<const uint32_t*>(&h01);
-      ph[kk][r + 1] = *reinterpret_cast<const uint32_t*>(&h23);
-    }
-    // O += P V with P in fp16 (11 significant bits; the row sum l uses the fp32 values) and V fp16
-    // (exactly the bf16-rounded values)
+      for (int j = 0; j < 4; ++j) {
+        const float p0 = exp2f(s[j][0] - ua), p1 = exp2f(s[j][1] - ua);
+        const float p2 = exp2f(s[j][2] - ub), p3 = exp2f(s[j][3] - ub);
+        l_a += p0 + p1;
+        l_b += p2 + p3;
+        const int kk = j >> 1, r = (j & 1) * 2;
+        const __half2 h01 = __floats2half2_rn(p0, p1), h23 = __floats2half2_rn(p2, p3);
+        ph[kk][r] = *reinterpret_cast<const uint32_t*>(&h01);
+        ph[kk][r + 1] = *reinterpret_cast<const uint32_t*>(&h23);
+      }
+      // O += P V with P in fp16 (11 significant bits; the row sum l uses the fp32 values) and V fp16
+      // (exactly the bf16-rounded values)
 #pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
+      for (int kk = 0; kk < 2; ++kk) {
 #pragma unroll
-      for (int dd = 0; dd < NDT / 2; ++dd) {
-        // trans matrices: (keys 16kk+0..7, dims 16dd+0..7), (keys +8..15, same), (keys 0..7, dims +8..15), (8..15, +8..15)
-        const int key = kk * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
-        const int ch = dd * 2 + (lane >> 4);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(vbase + kv_off<HD>(key, ch), b0, b1, b2, b3);
-        mma_f16_16816(o[2 * dd], ph[kk], b0, b1);
-        mma_f16_16816(o[2 * dd + 1], ph[kk], b2, b3);
+        for (int dd = 0; dd < NDT / 2; ++dd) {
+          // trans matrices: (keys 16kk+0..7, dims 16dd+0..7), (keys +8..15, same), (keys 0..7, dims +8..15), (8..15, +8..15)
+          const int key = hk * 32 + kk * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
+          const int ch = dd * 2 + (lane >> 4);
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(vbase + kv_off<HD>(key, ch), b0, b1, b2, b3);
+          mma_f16_16816(o[2 * dd], ph[kk], b0, b1);
+          mma_f16_16816(o[2 * dd + 1], ph[kk], b2, b3);
+        }
       }
     }
     named_bar_sync(bar_id, 128);  // buffer `buf` may be refilled next iteration
