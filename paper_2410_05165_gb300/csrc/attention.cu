@@ -100,7 +100,7 @@ bool attn_make_maps(const __nv_bfloat16* k_cache, const __half* v_cache, int row
   const int boxw = head_dim >= 64 ? 64 : head_dim;
   cuuint64_t dims[2] = {(cuuint64_t)d_model, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)d_model * 2};
-  cuuint32_t box[2] = {(cuuint32_t)boxw, (cuuint32_t)ATT_PAGE};
+  cuuint32_t box[2] = {(cuuint32_t)boxw, (cuuint32_t)ATT_SUB};
   cuuint32_t es[2] = {1, 1};
   const CUtensorMapSwizzle sw = head_dim >= 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE;
   for (int i = 0; i < 2; ++i) {

@@ -14,6 +14,7 @@
 namespace atspeed {
 
 constexpr int ATT_PAGE = 64;       // rows per KV page
+constexpr int ATT_SUB = 32;        // rows per K / V copy of the attention (half a page)
 constexpr int ATT_QTILE = 64;      // queries per CTA
 constexpr int ATT_MAX_ANC = 4;     // path keys per query (L = 4)
 

@@ -40,26 +40,32 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Byte offset of (row, 16-byte chunk) inside a K or V page tile as written by TMA.
+// Byte offset of (row, 16-byte chunk) inside a K or V tile of ATT_SUB rows as written by TMA.
 // HD >= 64: boxes of 64 columns (128 B rows), 128-byte swizzle: chunk ^= row & 7.
 // HD == 32: one box of 64-byte rows, no swizzle.
 template <int HD>
 __device__ __forceinline__ uint32_t kv_off(int row, int chunk16) {
   if constexpr (HD >= 64) {
     const int box = chunk16 >> 3, c = chunk16 & 7;
-    return (uint32_t)(box * (ATT_PAGE * 128) + row * 128 + ((c ^ (row & 7)) << 4));
+    return (uint32_t)(box * (ATT_SUB * 128) + row * 128 + ((c ^ (row & 7)) << 4));
   } else {
     return (uint32_t)(row * (HD * 2) + (chunk16 << 4));
   }
 }
 
+// Physical 16-byte chunk of logical chunk c of Q row r (conflict-free ldmatrix without padding).
+template <int HD>
+__device__ __forceinline__ int q_chunk(int r, int c) {
+  return c ^ (r & ((HD / 8 < 8 ? HD / 8 : 8) - 1));
+}
+
 template <int HD>
 struct AttCfg {
-  // SMEM_BODY: bytes from the 1024-aligned base: the K/V double buffer; the Q tile is staged in the
-  // second buffer before its first K/V copy (Q lives in registers from then on)
-  static constexpr int QSTRIDE = HD + 8;                    // bf16 elements per Q row in smem
-  static constexpr int Q_BYTES = ATT_QTILE * QSTRIDE * 2;
-  static constexpr int KV_BYTES = ATT_PAGE * HD * 2;         // one K (or V) page tile
+  // SMEM_BODY: bytes from the 1024-aligned base: the K/V double buffer (half pages of ATT_SUB keys);
+  // the Q tile (rows of HD bf16, 16-byte chunks XOR-swizzled by row) is staged in the second
+  // buffer before its first K/V copy (Q lives in registers from then on)
+  static constexpr int Q_BYTES = ATT_QTILE * HD * 2;
+  static constexpr int KV_BYTES = ATT_SUB * HD * 2;          // one K (or V) half-page tile
   static constexpr int BUF_BYTES = 2 * KV_BYTES;             // K + V
   static constexpr int SMEM_BODY = 2 * BUF_BYTES;
   static_assert(Q_BYTES <= BUF_BYTES, "the Q tile must fit in one K/V buffer");
@@ -103,18 +109,21 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
   const int* ptab = a.page_table + (size_t)u * a.max_pages;
   constexpr int NBOX = HD >= 64 ? HD / 64 : 1;
   constexpr int BOXW = HD >= 64 ? 64 : HD;
-  int c0 = 0, c1 = 0;   // this item's prefix chunks: thread 0 computes them, the others read s_info
-  int page1 = 0;        // page of the second chunk, loaded together with the first one's (thread 0)
-  auto issue = [&](int chunk, int buf) {
-    const int row0 = (chunk == c0 + 1 ? page1 : ptab[chunk]) * ATT_PAGE;
+  int c0 = 0, c1 = 0;   // this item's prefix pages: thread 0 computes them, the others read s_info
+  int page0 = 0, page1 = 0;   // cache pages of the first two pages (thread 0)
+  // copy of half page sc (keys sc * ATT_SUB ...) into buffer buf
+  auto issue = [&](int sc, int buf) {
+    const int pg = sc / (ATT_PAGE / ATT_SUB);
+    const int row0 = (pg == c0 ? page0 : pg == c0 + 1 ? page1 : ptab[pg]) * ATT_PAGE + (sc % (ATT_PAGE / ATT_SUB)) * ATT_SUB;
     uint8_t* kb = kvbuf + buf * C::BUF_BYTES;
     mbar_arrive_expect_tx(&bars[buf], C::BUF_BYTES);
     const uint64_t pol = policy_evict_last();
     for (int b = 0; b < NBOX; ++b) {
-      tma_load_2d(kb + b * (ATT_PAGE * BOXW * 2), mk, &bars[buf], h * HD + b * BOXW, row0, pol);
-      tma_load_2d(kb + C::KV_BYTES + b * (ATT_PAGE * BOXW * 2), mv, &bars[buf], h * HD + b * BOXW, row0, pol);
+      tma_load_2d(kb + b * (ATT_SUB * BOXW * 2), mk, &bars[buf], h * HD + b * BOXW, row0, pol);
+      tma_load_2d(kb + C::KV_BYTES + b * (ATT_SUB * BOXW * 2), mv, &bars[buf], h * HD + b * BOXW, row0, pol);
     }
   };
+  constexpr int SUBS = ATT_PAGE / ATT_SUB;
   if (tid == 0) {
     const int mv_ = max(max(s_info[2], s_info[3]), max(s_info[4], s_info[5]));
     const int nch = (mv_ + ATT_PAGE - 1) / ATT_PAGE;
@@ -125,10 +134,11 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
     }
     s_info[0] = c0;
     s_info[1] = c1;
-    // the first K / V chunk does not depend on Q: start its copy now
+    // the first K / V half page does not depend on Q: start its copy now
     if (c0 < c1) {
+      page0 = ptab[c0];
       if (c0 + 1 < c1) page1 = ptab[c0 + 1];
-      issue(c0, 0);
+      issue(c0 * SUBS, 0);
     }
   }
   // Q tile -> shared memory (rows >= nq are zero); all of a thread's loads are issued first
@@ -146,7 +156,7 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
     for (int k = 0; k < NQL; ++k) {
       const int i = tid + 128 * k;
       const int r = i / (HD / 8), c = i % (HD / 8);
-      *reinterpret_cast<uint4*>(qs + r * C::QSTRIDE + c * 8) = v[k];
+      *reinterpret_cast<uint4*>(qs + r * HD + q_chunk<HD>(r, c) * 8) = v[k];
     }
   }
   named_bar_sync(bar_id, 128);
@@ -159,10 +169,11 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
   {
     const uint32_t qbase = smem_u32(qs);
     const int r = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-    const int cofs = (lane >> 4) * 8;
+    const int cofs = lane >> 4;   // 16-byte chunk within the 16-column k-step
 #pragma unroll
     for (int kk = 0; kk < NKS; ++kk)
-      ldsm_x4(qbase + (uint32_t)((r * C::QSTRIDE + kk * 16 + cofs) * 2), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
+      ldsm_x4(qbase + (uint32_t)((r * HD + q_chunk<HD>(r, kk * 2 + cofs) * 8) * 2), qf[kk][0], qf[kk][1], qf[kk][2],
+              qf[kk][3]);
   }
   named_bar_sync(bar_id, 128);   // every warp holds its Q fragments: buffer 1 may receive K/V now
   const int g = lane >> 2, tq = lane & 3;
@@ -177,11 +188,11 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
   float m_a = -INFINITY, m_b = -INFINITY, l_a = 0.f, l_b = 0.f;
   bool ok = true;
 
-  for (int chunk = c0; chunk < c1; ++chunk) {
-    const int buf = (chunk - c0) & 1;
-    if (tid == 0 && chunk + 1 < c1) issue(chunk + 1, buf ^ 1);
+  for (int sc = c0 * SUBS; sc < c1 * SUBS; ++sc) {
+    const int buf = (sc - c0 * SUBS) & 1;
+    if (tid == 0 && sc + 1 < c1 * SUBS) issue(sc + 1, buf ^ 1);
     const bool got = named_bar_and(bar_id, 128, mbar_wait(&bars[buf], (uint32_t)(use[buf] & 1), a.err));
-    if (chunk - c0 < 2) ATT_TR(2 + 2 * (chunk - c0));
+    if (sc - c0 * SUBS < 2) ATT_TR(2 + 2 * (sc - c0 * SUBS));
     ++use[buf];
     if (!got) {
       ok = false;
@@ -189,9 +200,8 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
     }
     const uint32_t kbase = smem_u32(kvbuf + buf * C::BUF_BYTES);
     const uint32_t vbase = kbase + C::KV_BYTES;
-    // the page's 64 keys in two halves of 32 (fewer live registers), online softmax over each
-#pragma unroll 1
-    for (int hk = 0; hk < ATT_PAGE / 32; ++hk) {
+    {
+      constexpr int hk = 0;   // the buffer holds the half page's ATT_SUB = 32 keys
       float s[4][4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
@@ -209,7 +219,7 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
         }
       }
       // scale, mask, online softmax (base 2)
-      const int kbase_idx = chunk * ATT_PAGE + hk * 32;
+      const int kbase_idx = sc * ATT_SUB;
       float mx_a = m_a, mx_b = m_b;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -268,7 +278,7 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
       }
     }
     named_bar_sync(bar_id, 128);  // buffer `buf` may be refilled next iteration
-    if (chunk - c0 < 2) ATT_TR(3 + 2 * (chunk - c0));
+    if (sc - c0 * SUBS < 2) ATT_TR(3 + 2 * (sc - c0 * SUBS));
   }
   if (!ok) {
     // the copy for the next chunk may still be in flight: wait for it (bounded) before returning

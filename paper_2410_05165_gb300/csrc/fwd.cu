@@ -36,7 +36,7 @@ constexpr int ITEM_ROWS_FWD = 1024;   // item-code rows of the LM head (4 levels
 
 template <int BN>
 struct FCfg {
-  static constexpr int SA = BN == 128 ? 5 : 4;   // weight stages
+  static constexpr int SA = BN == 128 ? 8 : 5;   // weight stages
   static constexpr int SB = BN == 128 ? 3 : 3;   // activation stages
   static constexpr int A_BYTES = GEMM_BM * 128;
   static constexpr int B_BYTES = BN * 128;
