@@ -376,7 +376,7 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
           acc[b] = (in && P[b] == 0) ? __ldcg(reinterpret_cast<const float4*>(p.dh + e)) : zero;
           Pm = max(Pm, P[b]);
         }
-#pragma unroll 2
+#pragma unroll 4
         for (int e = 0; e < Pm; ++e) {
           float4 v[4];
 #pragma unroll
