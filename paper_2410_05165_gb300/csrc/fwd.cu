@@ -323,6 +323,14 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
     const int src = mode == 2 ? p.out_rows[r] : r;
     float* hr = p.h + (size_t)src * d;
     float ss = 0.f;
+    // the gains do not depend on the row: their loads go out with the first pass's
+    constexpr int NG_MAX = 8192 / 4 / CT;   // chunks per thread, d <= 8192
+    uint2 graw[NG_MAX];
+#pragma unroll
+    for (int k = 0; k < NG_MAX; ++k) {
+      const int c = ctid + CT * k;
+      graw[k] = c < nc ? *reinterpret_cast<const uint2*>(g + 4 * c) : make_uint2(0, 0);
+    }
     if (mode == 0) {
       const __nv_bfloat16* er = p.embed + (size_t)p.tok[r] * d;
       for (int k0 = 0; k0 * CT < nc; k0 += NORM_NB) {
@@ -419,11 +427,12 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
     if (p.trace && ctid == 0 && r == (int)blockIdx.x) p.trace[((size_t)5 * (7 * p.L + 2) + ph) * p.G + blockIdx.x] = globaltimer_ns();
     const float rs = 1.0f / sqrtf(rms_total(red) / (float)d + p.eps);
     __nv_bfloat16* xr = p.x + (size_t)r * d;
-#pragma unroll 4
-    for (int c = ctid; c < nc; c += CT) {
+#pragma unroll
+    for (int k = 0; k < NG_MAX; ++k) {
+      const int c = ctid + CT * k;
+      if (c >= nc) break;
       const float4 v = rowbuf[c];
-      const uint2 graw = *reinterpret_cast<const uint2*>(g + 4 * c);
-      const __nv_bfloat162* gb = reinterpret_cast<const __nv_bfloat162*>(&graw);
+      const __nv_bfloat162* gb = reinterpret_cast<const __nv_bfloat162*>(&graw[k]);
       const float2 g0 = __bfloat1622float2(gb[0]), g1 = __bfloat1622float2(gb[1]);
       __nv_bfloat162 o[2];
       o[0] = __floats2bfloat162_rn(v.x * rs * g0.x, v.y * rs * g0.y);
