@@ -243,10 +243,13 @@ def test_sd_strict_lossless_and_matches_oracle_tiny(ats):
             lambda ps: [ev.logits([p])[0][256 * len(p):256 * (len(p) + 1)].astype(np.float32) for p in ps],
             trie, w.K)
         got = [tuple(int(c) for c in r) for r in sd_items[u].cpu().numpy()]
-        np.testing.assert_allclose(sd_sc[u].cpu().numpy(), ref_sc, atol=2e-2)
+        # a beam score is the sum of its L = 4 levels' log-probs (Alg. 1), each within 2e-2 of the
+        # oracle's: the score within L x 2e-2, and a ranking may differ only across a gap below it
+        tol = 4 * 2e-2
+        np.testing.assert_allclose(sd_sc[u].cpu().numpy(), ref_sc, atol=tol)
         if got != ref:
             gaps = np.abs(np.diff(ref_sc.astype(np.float64)))
-            assert gaps.min() < 2e-2, (got, ref)
+            assert gaps.min() < tol, (got, ref)
     ctx.close()
 
 
