@@ -38,6 +38,7 @@ struct Fail {
 struct ModelRt {
   bool present = false;
   bool per_op = false;   // this model's forward runs one kernel per op (else one persistent launch)
+  int grid = 0;          // CTAs of its GEMM work splits (both schedules, so both give the same bits)
   int layers = 0, d = 0, H = 0, hd = 0, ffn = 0, V = 0;
   float eps = 1e-6f, theta = 1e4f;
   const bf16 *embed = nullptr, *final_norm = nullptr, *lm_head = nullptr;
@@ -136,7 +137,7 @@ struct atspeed_ctx {
   std::vector<ProfRec> prof_recs;
   std::vector<cudaEvent_t> prof_pool;
   long long n_launch = 0;  // kernels launched by this context (all kinds)
-  int forward_mode = 0;    // ATSPEED_FORWARD: 0 by model size, 1 persistent, 2 one kernel per op
+  int forward_mode = 0;    // ATSPEED_FORWARD: 0 default (persistent), 1 persistent, 2 one kernel per op
   int fwd_grid = 0;
   unsigned int* fwd_bar = nullptr;
   int* fwd_sk = nullptr;     // split-tile arrival counters of the persistent forward
@@ -490,13 +491,13 @@ struct ProfScope {
   }
 };
 
-void gemm(atspeed_ctx* c, const GemmArgs& a, cudaStream_t st, int kind) {
+void gemm(atspeed_ctx* c, const GemmArgs& a, cudaStream_t st, int kind, int grid) {
   char eb[256] = {0};
   // algorithmic bytes: weights once, activations in, outputs out
   const double out_b = a.epi == EPI_F32 ? 4.0 * a.M : a.epi == EPI_RESID ? 8.0 * a.M
                        : a.epi == EPI_SWIGLU ? 1.0 * a.M : 2.0 * a.M;
   ProfScope ps(c, st, kind, 2.0 * a.M * a.K + 2.0 * a.T * a.K + out_b * a.T, 2.0 * a.M * a.K * a.T);
-  cudaError_t e = gemm_launch(a, c->gs, c->gemm_grid, st, c->pdl && !c->prof, eb, sizeof eb);
+  cudaError_t e = gemm_launch(a, c->gs, grid, st, c->pdl && !c->prof, eb, sizeof eb);
   c->n_launch += 1;
   if (e != cudaSuccess) {
     set_err(c, "gemm launch failed: %s %s", cudaGetErrorString(e), eb);
@@ -537,7 +538,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     f.ffn = m.ffn;
     f.L = m.layers;
     f.eps = m.eps;
-    f.G = c->fwd_grid;
+    f.G = m.grid;
     f.maps = m.maps;
     f.attn_norm = m.d_attn_norm;
     f.mlp_norm = m.d_mlp_norm;
@@ -623,7 +624,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.q_out = m.q;
     g.k_cache = m.kc + per * l;
     g.v_cache = m.vc + per * l;
-    gemm(c, g, st, 0);
+    gemm(c, g, st, 0, m.grid);
     AttnArgs a = {};
     a.T = T;
     a.n_heads = m.H;
@@ -666,7 +667,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.X_rows = m.Xrows;
     g.out_f32 = m.h;
     g.ldo = m.d;
-    gemm(c, g, st, 1);
+    gemm(c, g, st, 1, m.grid);
     CK(rmsnorm_launch(m.h, nullptr, nullptr, nullptr, m.mlp_norm[l], T, m.d, m.eps, m.x, m.d, st, pdl));
     c->n_launch += 1;
     g = GemmArgs{};
@@ -679,7 +680,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.X_rows = m.Xrows;
     g.out_bf16 = m.act;
     g.ldo = m.ffn;
-    gemm(c, g, st, 2);
+    gemm(c, g, st, 2, m.grid);
     g = GemmArgs{};
     g.epi = EPI_RESID;
     g.W = m.wdown[l];
@@ -690,7 +691,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.X_rows = m.Xrows;
     g.out_f32 = m.h;
     g.ldo = m.d;
-    gemm(c, g, st, 3);
+    gemm(c, g, st, 3, m.grid);
   }
   const int n_out = (int)p.out_rows.size();
   CK(rmsnorm_rows_launch(m.h, m.rows_sel, n_out, m.final_norm, m.d, m.eps, m.x, m.d, st, pdl));
@@ -705,7 +706,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
   g.X_rows = m.Xrows;
   g.out_f32 = m.logits + (size_t)p.logit_row_base * ITEM_ROWS;
   g.ldo = ITEM_ROWS;
-  gemm(c, g, st, 4);
+  gemm(c, g, st, 4, m.grid);
 }
 
 void add_qtiles(FwdPlan& p, int u, int t0, int n) {
@@ -1209,15 +1210,16 @@ atspeed_status atspeed_create(const atspeed_model_desc* target, const atspeed_mo
     c->gemm_grid = gemm_grid_size(c->device);
     c->fwd_grid = c->gemm_grid;  // one persistent CTA per SM
     {
-      // Schedule of a model's forward: one persistent launch for models whose layer weights reach
-      // 1 GB (the weight stream then dwarfs the phase latencies), one kernel per op below that (a
-      // few-layer draft model, where the per-op kernels' shorter phases win).  ATSPEED_FORWARD=
-      // persistent | per_op forces one schedule for both models.
+      // Schedule of a model's forward: one persistent launch; ATSPEED_FORWARD=per_op runs one kernel
+      // per op instead (same bits).  GEMM work splits run over min(SMs, gate/up weight tiles) CTAs:
+      // a small model (the 4-layer draft: 48 tiles) then takes one whole gate/up tile per CTA with
+      // no split sums, and every phase's grid barrier spans fewer CTAs; a 7B-shape model (172 tiles)
+      // takes the whole GPU.
       const char* fm = getenv("ATSPEED_FORWARD");
       c->forward_mode = (fm && strcmp(fm, "persistent") == 0) ? 1 : (fm && strcmp(fm, "per_op") == 0) ? 2 : 0;
       for (ModelRt* mr : {&c->tgt, &c->drf}) {
-        const double wbytes = 2.0 * mr->layers * (4.0 * mr->d * mr->d + 3.0 * mr->d * mr->ffn);
-        mr->per_op = c->forward_mode == 2 || (c->forward_mode == 0 && wbytes < 1e9);
+        mr->per_op = c->forward_mode == 2;
+        mr->grid = std::max(1, std::min(c->fwd_grid, 2 * mr->ffn / 128));
       }
     }
     c->fwd_bar = dalloc<unsigned int>(c, 1);
