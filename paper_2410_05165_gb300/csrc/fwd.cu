@@ -117,7 +117,7 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
   g.m_tiles = (g.epi == EPI_SWIGLU) ? g.M / GEMM_BM : (g.M + GEMM_BM - 1) / GEMM_BM;
   g.n_tiles = (g.rows + BN - 1) / BN;
   g.kb = g.K / GEMM_BK;
-  g.w = work_split(g.m_tiles * g.n_tiles, g.kb, p.G);
+  g.w = work_split(g.m_tiles * g.n_tiles, g.kb, gemm_work_ctas((long long)g.m_tiles * g.n_tiles, g.kb, p.G));
   return g;
 }
 

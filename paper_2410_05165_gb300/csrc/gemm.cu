@@ -416,8 +416,7 @@ cudaError_t gemm_launch(const GemmArgs& a, const GemmScratch& s, int grid, cudaS
     snprintf(eb, el, "gemm: %lld tiles exceed the counter table (%d)", tiles, s.max_tiles);
     return cudaErrorInvalidValue;
   }
-  const long long U = tiles * kp.kb;
-  kp.G = (int)((long long)grid < U ? grid : U);
+  kp.G = gemm_work_ctas(tiles, kp.kb, grid);
   kp.w = work_split((int)tiles, kp.kb, kp.G);
   if (s.ws_bytes < gemm_ws_bytes(kp.G)) {
     snprintf(eb, el, "gemm: workspace too small");

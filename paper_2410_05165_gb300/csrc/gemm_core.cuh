@@ -19,6 +19,7 @@ struct WorkSplit {
   int tiles, kb, q, r;
   long long Usk;   // stream-K units: r * kb
   int Gsk;         // CTAs that get stream-K units: min(G, Usk)
+  int G;           // CTAs that take work (any others of the grid idle in this GEMM)
 };
 
 __host__ __device__ inline WorkSplit work_split(int tiles, int kb, int G) {
@@ -29,7 +30,20 @@ __host__ __device__ inline WorkSplit work_split(int tiles, int kb, int G) {
   w.r = tiles - w.q * G;
   w.Usk = (long long)w.r * kb;
   w.Gsk = (int)(w.Usk < (long long)G ? w.Usk : (long long)G);
+  w.G = G;
   return w;
+}
+
+// CTAs that take work in a GEMM of `tiles` tiles of kb k-blocks on a grid of `grid` CTAs.  With
+// fewer tiles than CTAs, the first `tiles` CTAs take one whole tile each (and the others idle) when
+// that costs at most 8 k-blocks more per CTA than spreading the k-blocks over the grid: every split
+// tile ends in a sum of its parts whose latency outweighs a short stream (a small model's QKV
+// projection).  Both the per-op GEMM and the persistent forward take their split from here, so
+// their sums are the same bit for bit.
+__host__ __device__ inline int gemm_work_ctas(long long tiles, int kb, int grid) {
+  if (tiles < grid && (long long)kb * (grid - tiles) <= 8LL * grid) return (int)tiles;
+  const long long U = tiles * kb;
+  return (int)(U < (long long)grid ? U : (long long)grid);
 }
 // stream-K unit range [a, b) of CTA c
 __device__ __forceinline__ void sk_range(const WorkSplit& w, int c, long long& a, long long& b) {
@@ -46,6 +60,7 @@ __device__ __forceinline__ int sk_owner(const WorkSplit& w, long long u) {
 }
 // number of units of CTA c, and its i-th unit as (tile, k-block)
 __device__ __forceinline__ long long cta_units(const WorkSplit& w, int c) {
+  if (c >= w.G) return 0;
   long long a, b;
   sk_range(w, c, a, b);
   return (b - a) + (long long)w.q * w.kb;
@@ -69,6 +84,11 @@ struct SegIter {
   long long u, u1;
   int dp, dp1;
   __device__ __forceinline__ void init(const WorkSplit& w, int c) {
+    if (c >= w.G) {
+      u = u1 = 0;
+      dp = dp1 = 0;
+      return;
+    }
     sk_range(w, c, u, u1);
     dp = w.r + c * w.q;
     dp1 = dp + w.q;
