@@ -72,6 +72,11 @@ def parse():
                     help="profiling aid for --verify-only: cut the target to its first L layers (small ncu captures)")
     ap.add_argument("--kernel-probe", action="store_true",
                     help="profiling aid: the four layer GEMMs of the 7B shape at T=120 over 8 layers of weights")
+    ap.add_argument("--sweep", action="store_true",
+                    help="verification-call sweep on the 7B-shape target (512-token prompts, 50 000 items): "
+                         "K in {1,5,10,20} x gamma in {1..4} x N in {K,2K,4K} x batch in {1,4,16}, strict and "
+                         "relaxed; one JSON line per point")
+    ap.add_argument("--sweep-batches", default="1,4,16", help="--sweep: the batch axis")
     return ap.parse_args()
 
 
@@ -426,9 +431,67 @@ def verify_only(w, mode, reps, layers=0):
     ctx.close()
 
 
+def sweep(batches, reps=2):
+    """Verification-call sweep: for every (batch, K, gamma, N, mode) point, prefill the batch's
+    512-token histories, draft gamma levels of width N and time the first verification call (median
+    of `reps`), with its tree-token count, roofline fraction and accepted steps per user."""
+    import torch
+    import paper_2410_05165_gb300 as ats
+    ats.load()
+    w = synth.workload("7b")
+    hbm, tf, _, src = peaks()
+    tw = {n: torch.from_numpy(a).to(device="cuda", dtype=torch.bfloat16)
+          for n, a in synth.iter_model_tensors(w.target, w.seed, "target")}
+    dw = {n: torch.from_numpy(a).to(device="cuda", dtype=torch.bfloat16)
+          for n, a in synth.iter_model_tensors(w.draft, w.seed, "draft")}
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    for B in batches:
+        prompts = synth.make_prompts(B, w.prompt_len, w.target.vocab, w.seed)
+        P = [len(p) for p in prompts]
+        ctx = ats.Context(w.target, tw, w.draft, dw, items, w.code_base, max_users=B, max_prompt=max(P),
+                          max_K=20, max_N=80, max_gamma=4)
+        toks = torch.from_numpy(np.concatenate(prompts).astype(np.int32)).cuda()
+        off = np.concatenate([[0], np.cumsum(P)]).astype(np.int32)
+        for K in (1, 5, 10, 20):
+            for gamma in (1, 2, 3, 4):
+                for N in (K, 2 * K, 4 * K):
+                    for mode in ("strict", "relaxed"):
+                        o = ats.opts(K, N, gamma, w.philox_seed)
+                        vm = ats.STRICT if mode == "strict" else ats.RELAXED
+                        ms, acc_mean, T = [], 0.0, 0
+                        for _ in range(reps):
+                            ctx.prefill(toks, off)
+                            ctx.begin_step(o)
+                            for _ in range(gamma):
+                                ctx.draft_step(o, vm)
+                            # tree tokens of the call: the drafted levels 1 .. min(gamma, L - 1) (level-L
+                            # nodes complete an item and are not forwarded; no incoming beams at depth 0)
+                            cnt = ctx.debug_tree(gamma)["count"]
+                            T = int(cnt[:, 1:1 + min(gamma, 3)].sum())
+                            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                            e0.record()
+                            acc, _, _, _ = ctx.verify(o, vm)
+                            e1.record()
+                            torch.cuda.synchronize()
+                            ms.append(e0.elapsed_time(e1))
+                            acc_mean = float(acc.float().mean())
+                        vb, vf = verify_bytes_flops(w, T, P)
+                        t_roof = max(vb / (hbm * 1e9), vf / (tf * 1e12)) * 1e3
+                        v = float(np.median(ms))
+                        print(json.dumps({"sweep": "verify", "batch": B, "K": K, "gamma": gamma, "N": N, "mode": mode,
+                                          "tree_tokens": T, "verify_ms": round(v, 4),
+                                          "bound": "hbm" if vb / (hbm * 1e9) >= vf / (tf * 1e12) else "tensor",
+                                          "roofline_frac": round(t_roof / v, 4), "accepted_steps": acc_mean,
+                                          "peak_source": src}), flush=True)
+        ctx.close()
+
+
 def main():
     args = parse()
     w = synth.workload(args.workload)
+    if args.sweep:
+        sweep([int(b) for b in args.sweep_batches.split(",")])
+        return
     if args.kernel_probe:
         kernel_probe()
         return

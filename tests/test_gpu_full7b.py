@@ -100,3 +100,23 @@ def test_7b_relaxed_outputs_are_valid_distinct_ranked(ats, world):
     assert stats[0, 1] >= 1
     del trie
     ctx.close()
+
+
+@pytest.mark.parametrize("B,K,gamma,N", [(4, 5, 2, 10), (1, 20, 3, 80), (4, 1, 4, 4)])
+def test_7b_sweep_points_strict_lossless(ats, world, B, K, gamma, N):
+    """Points of the verification-call sweep (batch x K x gamma x N, 512-token histories): strict
+    speculative decoding returns the plain target beam search's lists bit for bit, for every user."""
+    w, _, _, items, _, _ = world
+    prompts = synth.make_prompts(B, w.prompt_len, w.target.vocab, w.seed + 7)
+    P = [len(p) for p in prompts]
+    ctx = ats.Context(w.target, world[1], w.draft, world[2], items, w.code_base, max_users=B, max_prompt=max(P),
+                      max_K=20, max_N=80, max_gamma=4)
+    toks = torch.from_numpy(np.concatenate(prompts).astype(np.int32)).cuda()
+    off = np.concatenate([[0], np.cumsum(P)]).astype(np.int32).tolist()
+    o = ats.opts(K, N, gamma, w.philox_seed)
+    sd_items, sd_sc, stats = ctx.beam_search(toks, off, o, ats.SD_STRICT)
+    pl_items, pl_sc, _ = ctx.beam_search(toks, off, o, ats.PLAIN_TOPK)
+    np.testing.assert_array_equal(sd_items.cpu().numpy(), pl_items.cpu().numpy())
+    np.testing.assert_array_equal(sd_sc.cpu().numpy(), pl_sc.cpu().numpy())
+    assert sd_items.shape == (B, K, 4)
+    ctx.close()
