@@ -255,14 +255,16 @@ def sd_decode(target_rows: RowsFn, draft_rows: RowsFn, trie, K: int, N: int, gam
 
 
 def plain_beam_search(target_rows: RowsFn, trie, K: int, L: int = 4, sample: bool = False, seed: int = 0,
-                      user: int = 0):
+                      user: int = 0, full_rows: Optional[RowsFn] = None):
     """Target-only constrained beam search (top-K), or sampling beam search at temperature 1.
 
     Sampling draws level l's K beams without replacement (Gumbel keys) from the Philox stream 3
-    counter with sd_step = l - 1, i.e. the number of steps taken before, as in the SD loop."""
+    counter with sd_step = l - 1, i.e. the number of steps taken before, as in the SD loop.
+    ``full_rows`` (the whole-vocabulary logit rows of the beams) selects FULL normalisation (O4):
+    each token's log-prob is normalised over the whole vocabulary, then masked to the trie."""
     beams, sp = [()], np.zeros(1, dtype=F32)
     for lvl in range(1, L + 1):
-        C = expand(beams, sp, target_rows(beams), trie)
+        C = expand(beams, sp, target_rows(beams), trie, None if full_rows is None else full_rows(beams))
         if sample:
             keys = (C.score + Philox(seed, lvl - 1, user).gumbel(STREAM_RESAMPLE, lvl, C.index)).astype(F32)
             sel = rank_order(keys, C.index)[:K]

@@ -120,3 +120,61 @@ def test_expand_candidate_order_and_scores():
     lp = constrained_logprobs(rows([(1,)])[0], np.array([2, 5]))
     np.testing.assert_array_equal(c.score[:2], (np.float32(-0.5) + lp).astype(np.float32))
     assert c.score[2] == np.float32(-1.0)   # single child: lp = 0
+
+
+def hashed_full_rows(item_rows, seed, extra=700, std=3.0):
+    """Whole-vocabulary rows consistent with ``item_rows``: the level's 256 code logits followed by
+    `extra` other token logits (hashed from the path)."""
+    def f(paths):
+        return [np.concatenate([r, (np.random.default_rng([seed, 77, len(p), *p]).standard_normal(extra) * std)
+                                .astype(np.float32)]) for p, r in zip(paths, item_rows(paths))]
+    return f
+
+
+def test_full_beam_search_equals_brute_force_when_exhaustive():
+    """FULL normalisation: an item's score is the fp32 sum of logit - logsumexp(whole row) over its
+    tokens; with every prefix kept, the beam search's list is the exact top-K over all items."""
+    rng = np.random.default_rng(6)
+    for trial in range(5):
+        items = np.unique(rng.integers(0, 256, size=(12, 4)), axis=0)
+        trie = Trie(items)
+        rows = hashed_rows(300 + trial)
+        full = hashed_full_rows(rows, 300 + trial)
+        beams, sp = plain_beam_search(rows, trie, 16, full_rows=full)
+        scores = []
+        for it in items:
+            s = 0.0
+            for lvl in range(4):
+                pre = tuple(int(c) for c in it[:lvl])
+                fr = full([pre])[0].astype(np.float64)
+                s += fr[int(it[lvl])] - scipy.special.logsumexp(fr)
+            scores.append(s)
+        scores = np.array(scores)
+        got = {tuple(int(c) for c in b): float(v) for b, v in zip(beams, sp)}
+        assert set(got) == {tuple(int(c) for c in it) for it in items}
+        for it, ref in zip(items, scores):
+            assert abs(got[tuple(int(c) for c in it)] - ref) < 1e-4
+        # ranking: scores descending
+        assert all(sp[i] >= sp[i + 1] for i in range(len(sp) - 1))
+
+
+def test_full_reduces_to_masked_when_the_row_holds_only_valid_children():
+    """A whole-vocabulary row whose only finite logits are the trie's valid children normalises
+    exactly as MASKED."""
+    rng = np.random.default_rng(8)
+    items = np.unique(rng.integers(0, 256, size=(40, 4)), axis=0)
+    trie = Trie(items)
+    rows = hashed_rows(500)
+
+    def full(paths):
+        out = []
+        for p, r in zip(paths, rows(paths)):
+            fr = np.full(256, -np.inf, dtype=np.float32)
+            kids = trie.children(p)
+            fr[kids] = r[kids]
+            out.append(fr)
+        return out
+    b_m, s_m = plain_beam_search(rows, trie, 5)
+    b_f, s_f = plain_beam_search(rows, trie, 5, full_rows=full)
+    assert b_m == b_f
+    np.testing.assert_allclose(s_f, s_m, atol=1e-5)
