@@ -66,6 +66,9 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="7b")
     ap.add_argument("--mode", choices=["strict", "relaxed"], default="strict")
+    ap.add_argument("--norm", choices=["masked", "full"], default="masked",
+                    help="constrained log-softmax normaliser: the valid children (default) or the whole "
+                         "vocabulary (the LM head then runs over all V rows)")
     ap.add_argument("--verify-only", type=int, default=0, metavar="R",
                     help="profiling aid: R verification calls of the workload, each in an NVTX range 'verify'")
     ap.add_argument("--layers", type=int, default=0, metavar="L",
@@ -96,14 +99,16 @@ def peaks():
         return 6800.0, 1900.0, 1700.0, "fallback"
 
 
-def verify_bytes_flops(w, T, P_users):
-    """Algorithmic bytes / FLOPs of one verification call: weights once, item-code LM-head rows,
-    every user's prefix KV read once, the tree's node KV written (bf16)."""
+def verify_bytes_flops(w, T, P_users, full=False):
+    """Algorithmic bytes / FLOPs of one verification call: weights once, item-code LM-head rows (all
+    V rows under FULL normalisation), every user's prefix KV read once, the tree's node KV written
+    (bf16)."""
     t = w.target
     d, f, Lr = t.d_model, t.d_ffn, t.n_layers
     per_layer = 4 * d * d + 3 * d * f
-    B = 2 * Lr * per_layer + 2 * 1024 * d + sum(P_users) * Lr * 2 * d * 2 + T * Lr * 2 * d * 2
-    F = 2 * T * Lr * per_layer + sum(4 * (T / len(P_users)) * (P + 2) * d * Lr for P in P_users) + 2 * T * d * 1024
+    head = t.vocab if full else 1024
+    B = 2 * Lr * per_layer + 2 * head * d + sum(P_users) * Lr * 2 * d * 2 + T * Lr * 2 * d * 2
+    F = 2 * T * Lr * per_layer + sum(4 * (T / len(P_users)) * (P + 2) * d * Lr for P in P_users) + 2 * T * d * head
     return B, F
 
 
@@ -243,7 +248,7 @@ def run_ours(args, w):
     h_tok = torch.from_numpy(np.concatenate(prompts).astype(np.int32)).pin_memory()
     toks = h_tok.cuda()
     offsets = np.concatenate([[0], np.cumsum(P_users)]).astype(np.int32)
-    o = ats.opts(w.K, w.N, w.gamma, w.philox_seed)
+    o = ats.opts(w.K, w.N, w.gamma, w.philox_seed, norm=ats.NORM_FULL if args.norm == "full" else ats.NORM_MASKED)
     stream = torch.cuda.current_stream()
 
     def barrier():
@@ -313,7 +318,7 @@ def run_ours(args, w):
         elif rep >= 3:
             ver_ms.append(e0.elapsed_time(e1))
     T_first = min(w.gamma, 3) * w.N * B
-    vb, vf = verify_bytes_flops(w, T_first, P_users)
+    vb, vf = verify_bytes_flops(w, T_first, P_users, full=args.norm == "full")
     v_ms = statistics.median(ver_ms)
     t_roof = max(vb / (hbm * 1e9), vf / (tf * 1e12)) * 1e3
     k_ms = fk["ms"] / max(1, fk["launches"])
@@ -333,7 +338,7 @@ def run_ours(args, w):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights, synthetic items)",
         "config": {"workload": f"{w.name}: 7B-shape target (32L d4096 H32 ffn11008 V33024), draft 4L d768, "
                                f"K={w.K} N={w.N} gamma={w.gamma}, P={w.prompt_len[0]}, {w.n_items} Zipf items, "
-                               f"{args.mode} verification, {B} user(s) per GPU",
+                               f"{args.mode} verification, {args.norm} normalisation, {B} user(s) per GPU",
                    "l2": "inputs larger than L2 (13.5 GB of target weights per verification call)"},
         "roofline": dict(roof, **{
             "traffic": TRAFFIC_PER_ALG_BYTE * vb,

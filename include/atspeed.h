@@ -92,7 +92,9 @@ typedef struct {
   int K;                  /* recommended items / target beam width          */
   int N;                  /* draft beam width                                */
   int gamma;              /* drafted beam-search steps per speculative step */
-  atspeed_norm_mode norm; /* only ATSPEED_NORM_MASKED in this build          */
+  atspeed_norm_mode norm; /* MASKED or FULL; fixed for a speculative step. FULL runs the LM
+                           * head over all V rows of every forwarded node (log-sum-exp
+                           * epilogue): V x d_model x 2 more weight bytes per forward      */
   uint64_t philox_seed;   /* key of the Philox4x32-10 streams (relaxed mode) */
 } atspeed_decode_opts;
 
@@ -181,7 +183,9 @@ atspeed_status atspeed_profile_read(atspeed_ctx *ctx, int kind, int32_t *h_launc
  * 3 attention output (bf16), 4 SwiGLU output (bf16 [T][d_ffn]), 5 K cache (bf16, all layers),
  * 6 V cache (fp16), 7 item-code logits (fp32 [rows][1024]), 8 the persistent forward's barrier
  * counter (u32), 9 its per-phase timestamps ([phases][CTAs] u64 ns, recorded only when the
- * environment variable ATSPEED_FWD_TRACE=1 was set at create time).  Synchronises the device. */
+ * environment variable ATSPEED_FWD_TRACE=1 was set at create time), 10 the whole-vocabulary
+ * log-sum-exp of each logits row (fp32 [rows], written under FULL normalisation).
+ * Synchronises the device. */
 atspeed_status atspeed_debug_buffer(atspeed_ctx *ctx, int which, int id, void *h_out, size_t bytes);
 
 /* Shape of the current speculative step: h_depth[n_users], h_levels[n_users] (drafted levels),
@@ -198,6 +202,11 @@ atspeed_status atspeed_debug_tree(atspeed_ctx *ctx, int32_t *h_path, float *h_sq
 /* Item-code logits [1024] of a node of the current step (which = 0 target, 1 draft), for the
  * node in slot `slot` of user `user`, copied to the host.  ATSPEED_E_STATE if it was not forwarded. */
 atspeed_status atspeed_debug_node_logits(atspeed_ctx *ctx, int which, int user, int slot, float *h_logits);
+
+/* Under FULL normalisation: the log-sum-exp over the whole vocabulary of the same node's logits row
+ * (which = 0 target, 1 draft), one float copied to the host.  ATSPEED_E_ARG outside a FULL step,
+ * ATSPEED_E_STATE if the node was not forwarded. */
+atspeed_status atspeed_debug_node_lse(atspeed_ctx *ctx, int which, int user, int slot, float *h_lse);
 
 /* Replaces the drafted tree of the current step (after prefill / a previous verify, before
  * verify): levels j = 1..n_levels, each with h_count[u*n_levels + j-1] nodes given as

@@ -25,7 +25,7 @@ EXPORTS = [
     "atspeed_create", "atspeed_destroy", "atspeed_last_error", "atspeed_prefill", "atspeed_begin_step",
     "atspeed_draft_step", "atspeed_verify", "atspeed_draft_step_logits", "atspeed_verify_logits",
     "atspeed_beam_search", "atspeed_profile", "atspeed_profile_read", "atspeed_tree_shape", "atspeed_debug_tree",
-    "atspeed_debug_node_logits", "atspeed_debug_buffer", "atspeed_set_tree", "atspeed_op_workspace_bytes", "atspeed_op_gemm",
+    "atspeed_debug_node_logits", "atspeed_debug_node_lse", "atspeed_debug_buffer", "atspeed_set_tree", "atspeed_op_workspace_bytes", "atspeed_op_gemm",
     "atspeed_op_gemm_noalloc", "atspeed_op_gemm_swiglu", "atspeed_op_rmsnorm", "atspeed_op_attention_scratch", "atspeed_op_attention",
 ]
 
@@ -92,6 +92,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "atspeed_tree_shape": (c_int, [vp, i32p, i32p, i32p, i32p]),
         "atspeed_debug_tree": (c_int, [vp, i32p, fp, fp, i32p]),
         "atspeed_debug_node_logits": (c_int, [vp, c_int, c_int, c_int, fp]),
+        "atspeed_debug_node_lse": (c_int, [vp, c_int, c_int, c_int, fp]),
         "atspeed_debug_buffer": (c_int, [vp, c_int, c_int, vp, ctypes.c_size_t]),
         "atspeed_set_tree": (c_int, [vp, vp, c_int, i32p, i32p, i32p, fp, fp]),
         "atspeed_op_workspace_bytes": (ctypes.c_size_t, []),
@@ -150,8 +151,8 @@ def _model_desc(spec, w: Dict[str, torch.Tensor]):
     return d, arrs
 
 
-def opts(K: int, N: int, gamma: int, seed: int = 0) -> DecodeOpts:
-    return DecodeOpts(K, N, gamma, NORM_MASKED, seed)
+def opts(K: int, N: int, gamma: int, seed: int = 0, norm: int = NORM_MASKED) -> DecodeOpts:
+    return DecodeOpts(K, N, gamma, norm, seed)
 
 
 class Context:
@@ -295,6 +296,12 @@ class Context:
         _check(self._lib.atspeed_debug_node_logits(self.ptr, which, user, slot,
                                                    out.ctypes.data_as(ctypes.POINTER(ctypes.c_float))), self.ptr)
         return out
+
+    def node_lse(self, which: int, user: int, slot: int) -> float:
+        out = np.zeros(1, np.float32)
+        _check(self._lib.atspeed_debug_node_lse(self.ptr, which, user, slot,
+                                                out.ctypes.data_as(ctypes.POINTER(ctypes.c_float))), self.ptr)
+        return float(out[0])
 
     def set_tree(self, counts: np.ndarray, parents: np.ndarray, codes: np.ndarray, sq: np.ndarray,
                  draft_logits: Optional[np.ndarray] = None, stream=None):

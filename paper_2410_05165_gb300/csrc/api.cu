@@ -57,6 +57,13 @@ struct ModelRt {
   bf16 *x = nullptr, *q = nullptr, *att = nullptr, *act = nullptr;
   float* logits = nullptr;  // [logit_rows][1024]
   int logit_rows = 0;
+  // FULL normalisation: whole-vocabulary log-sum-exp per logits row, the LM head's per-tile
+  // partials [ceil(V / 128)][lse_ld], and the prefill's final-norm rows of the last history tokens
+  float* lse = nullptr;
+  float2* lse_part = nullptr;
+  int lse_ld = 0;
+  bf16* root_x = nullptr;
+  int root_rows = 0;
   // per-token forward inputs
   int *tok = nullptr, *pos = nullptr, *kvrow = nullptr, *tuser = nullptr, *tvis = nullptr, *anc = nullptr,
       *ancn = nullptr;
@@ -120,6 +127,7 @@ struct atspeed_ctx {
   int B = 0;
   bool prefilled = false;
   bool step_open = false;      // level 0 of the current step is on the device
+  bool full_norm = false;      // the current step normalises over the whole vocabulary (FULL)
   int step_K = 0, step_N = 0, step_gamma = 0, levels_done = 0;
   bool roots_drafted = false;
   bool tree_injected = false;
@@ -293,6 +301,11 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.act = dalloc<bf16>(c, (size_t)m.Xrows * m.ffn);
   m.logit_rows = L.max_users + L.max_users * stride;
   m.logits = dalloc<float>(c, (size_t)m.logit_rows * ITEM_ROWS);
+  m.lse = dalloc<float>(c, m.logit_rows);
+  m.lse_ld = m.Tcap;
+  m.lse_part = dalloc<float2>(c, (size_t)((m.V + 127) / 128) * m.lse_ld, false);
+  m.root_rows = ((L.max_users + 255) / 256) * 256;
+  m.root_x = dalloc<bf16>(c, (size_t)m.root_rows * m.d);
   m.tok = dalloc<int>(c, m.Tcap);
   m.pos = dalloc<int>(c, m.Tcap);
   m.kvrow = dalloc<int>(c, m.Tcap);
@@ -438,6 +451,8 @@ TreeDev tree_dev(atspeed_ctx* c) {
   t.trie_child = c->trie_child;
   t.logits_t = c->tgt.logits;
   t.logits_d = c->drf.present ? c->drf.logits : c->tgt.logits;
+  t.lse_t = c->full_norm ? c->tgt.lse : nullptr;
+  t.lse_d = c->full_norm ? (c->drf.present ? c->drf.lse : c->tgt.lse) : nullptr;
   return t;
 }
 
@@ -709,6 +724,30 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
   gemm(c, g, st, 4, m.grid);
 }
 
+// FULL normalisation (whole-vocabulary log-softmax, then the trie mask): log-sum-exp over the whole
+// vocabulary of the n final-norm rows X[0 .. n) (bf16, X_rows allocated) into lse_out[0 .. n): the
+// LM head over all V rows with the EPI_LSE epilogue, then the combine of its per-tile partials.
+void full_lse(atspeed_ctx* c, ModelRt& m, const bf16* X, int X_rows, int n, float* lse_out, cudaStream_t st) {
+  if (n <= 0) return;
+  if (n > m.lse_ld) {
+    set_err(c, "FULL normalisation of %d rows exceeds the partials buffer (%d)", n, m.lse_ld);
+    throw Fail{ATSPEED_E_SHAPE};
+  }
+  GemmArgs g = {};
+  g.epi = EPI_LSE;
+  g.W = m.lm_head;
+  g.X = X;
+  g.M = m.V;
+  g.K = m.d;
+  g.T = n;
+  g.X_rows = X_rows;
+  g.lse_part = m.lse_part;
+  g.lse_ld = m.lse_ld;
+  gemm(c, g, st, 4, m.grid);
+  CK(lse_combine_launch(m.lse_part, m.lse_ld, (m.V + 127) / 128, n, lse_out, st));
+  c->n_launch += 1;
+}
+
 void add_qtiles(FwdPlan& p, int u, int t0, int n) {
   for (int i = 0; i < n; i += ATT_QTILE) {
     p.qt_t0.push_back(t0 + i);
@@ -751,6 +790,7 @@ void forward_nodes(atspeed_ctx* c, ModelRt& m, bool target, const std::vector<in
   for (int k = 0; k < T; ++k) p.out_rows[k] = k;
   p.logit_row_base = row_base;
   forward(c, m, p, st);
+  if (c->full_norm) full_lse(c, m, m.x, m.Xrows, T, m.lse + row_base, st);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -827,6 +867,15 @@ void open_step(atspeed_ctx* c, const atspeed_decode_opts* o, cudaStream_t st) {
   CK(cudaMemcpyAsync(c->n_sq, sq.data(), n * 4, cudaMemcpyHostToDevice, st));
   CK(cudaMemcpyAsync(c->n_sp, sp.data(), n * 4, cudaMemcpyHostToDevice, st));
   CK(cudaMemcpyAsync(c->n_cnt, cnt.data(), cnt.size() * 4, cudaMemcpyHostToDevice, st));
+  c->full_norm = o->norm == ATSPEED_NORM_FULL;
+  if (c->full_norm) {
+    // level 0 of users at depth 0 scores with the prefill's logits rows 0 .. B-1
+    bool fresh = false;
+    for (int u = 0; u < c->B; ++u) fresh |= c->users[u].active && c->users[u].d == 0;
+    if (fresh)
+      for (ModelRt* m : {&c->tgt, &c->drf})
+        if (m->present) full_lse(c, *m, m->root_x, m->root_rows, c->B, m->lse, st);
+  }
   upload_users(c, st);  // synchronises (host vectors above are local)
   c->step_open = true;
   c->have_tree = true;
@@ -846,15 +895,19 @@ void check_opts(atspeed_ctx* c, const atspeed_decode_opts* o) {
             o->gamma, c->lim.max_K, c->lim.max_N, c->lim.max_gamma);
     throw Fail{ATSPEED_E_SHAPE};
   }
-  if (o->norm != ATSPEED_NORM_MASKED) {
-    set_err(c, "only ATSPEED_NORM_MASKED is implemented");
-    throw Fail{ATSPEED_E_UNSUPPORTED};
+  if (o->norm != ATSPEED_NORM_MASKED && o->norm != ATSPEED_NORM_FULL) {
+    set_err(c, "unknown normalisation mode %d", (int)o->norm);
+    throw Fail{ATSPEED_E_ARG};
   }
 }
 
 void ensure_step(atspeed_ctx* c, const atspeed_decode_opts* o, cudaStream_t st) {
   if (!c->prefilled) {
     set_err(c, "prefill must come first");
+    throw Fail{ATSPEED_E_STATE};
+  }
+  if (c->step_open && (o->norm == ATSPEED_NORM_FULL) != c->full_norm) {
+    set_err(c, "the normalisation mode cannot change within a speculative step");
     throw Fail{ATSPEED_E_STATE};
   }
   if (!c->step_open) open_step(c, o, st);
@@ -1056,6 +1109,8 @@ void prefill_impl(atspeed_ctx* c, cudaStream_t st, int n_users, const int32_t* d
     CK(cudaMemcpyAsync(m->tuser, tuser.data(), T * 4, cudaMemcpyHostToDevice, st));
     CK(cudaMemcpyAsync(m->tvis, tvis.data(), T * 4, cudaMemcpyHostToDevice, st));
     forward(c, *m, p, st);
+    // the last history tokens' final-norm rows, for a FULL-normalised first step
+    CK(cudaMemcpyAsync(m->root_x, m->x, (size_t)n_users * m->d * sizeof(bf16), cudaMemcpyDeviceToDevice, st));
   }
   std::vector<int> Pu(P);
   CK(cudaMemcpyAsync(c->u_P, Pu.data(), n_users * 4, cudaMemcpyHostToDevice, st));
@@ -1101,6 +1156,10 @@ void draft_step_logits_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decod
   }
   const int off = lvl == 1 ? 0 : c->step_K + (lvl - 2) * c->step_N;
   const int width = lvl == 1 ? c->step_K : c->step_N;
+  if (c->full_norm) {
+    set_err(c, "injected logits carry no whole-vocabulary rows: FULL normalisation needs forwarded nodes");
+    throw Fail{ATSPEED_E_STATE};
+  }
   inject_logits(c, false, off, width, h_logits, (size_t)width * ITEM_ROWS, st);
   const TreeDev t = tree_dev(c);
   CK(draft_level_launch(t, lvl, c->step_N, mode == ATSPEED_RELAXED, o->philox_seed, st, c->pdl));
@@ -1123,6 +1182,10 @@ void verify_logits_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_op
     if (us.active && c->levels_done < us.g && !c->tree_injected) us.g = c->levels_done;
   }
   upload_users(c, st);
+  if (c->full_norm) {
+    set_err(c, "injected logits carry no whole-vocabulary rows: FULL normalisation needs forwarded nodes");
+    throw Fail{ATSPEED_E_STATE};
+  }
   inject_logits(c, true, 0, stride, h_logits, (size_t)stride * ITEM_ROWS, st);
   const TreeDev t = tree_dev(c);
   VerifyOut vo{c->o_acc, c->o_adv, c->o_n, c->o_nacc, c->o_path, c->o_score, c->o_parent, c->o_trie};
@@ -1466,6 +1529,7 @@ atspeed_status atspeed_debug_buffer(atspeed_ctx* c, int which, int id, void* h_o
       case 7: src = m.logits; cap = (size_t)m.logit_rows * ITEM_ROWS * 4; break;
       case 8: src = c->fwd_bar; cap = 4; break;
       case 9: src = c->fwd_trace; cap = c->fwd_trace_n * 8; break;
+      case 10: src = m.lse; cap = (size_t)m.logit_rows * 4; break;
       default: break;
     }
     if (!m.present || !src || !h_out || bytes > cap) {
@@ -1521,6 +1585,26 @@ atspeed_status atspeed_debug_node_logits(atspeed_ctx* c, int which, int user, in
     }
     const ModelRt& m = which == 0 ? c->tgt : c->drf;
     CK(cudaMemcpy(h_logits, m.logits + (size_t)row * ITEM_ROWS, ITEM_ROWS * 4, cudaMemcpyDeviceToHost));
+  });
+}
+
+atspeed_status atspeed_debug_node_lse(atspeed_ctx* c, int which, int user, int slot, float* h_lse) {
+  return guarded(c, [&] {
+    const int stride = c->step_K + c->step_gamma * c->step_N;
+    if (!c->have_tree || !c->full_norm || user < 0 || user >= c->B || slot < 0 || slot >= stride || !h_lse) {
+      set_err(c, "debug_node_lse: bad arguments, no open step or not a FULL-normalised step");
+      throw Fail{ATSPEED_E_ARG};
+    }
+    CK(cudaDeviceSynchronize());
+    int row = -1;
+    CK(cudaMemcpy(&row, (which == 0 ? c->n_lg_t : c->n_lg_d) + (size_t)user * stride + slot, 4,
+                  cudaMemcpyDeviceToHost));
+    if (row < 0) {
+      set_err(c, "node was not forwarded");
+      throw Fail{ATSPEED_E_STATE};
+    }
+    const ModelRt& m = (which == 0 || !c->drf.present) ? c->tgt : c->drf;
+    CK(cudaMemcpy(h_lse, m.lse + row, 4, cudaMemcpyDeviceToHost));
   });
 }
 

@@ -366,11 +366,32 @@ cudaError_t launch_bn(EpiKind e, const CUtensorMap& ma, const CUtensorMap& mb, c
     case EPI_RESID: return launch_t<BN, EPI_RESID>(ma, mb, kp, st, pdl);
     case EPI_SWIGLU: return launch_t<BN, EPI_SWIGLU>(ma, mb, kp, st, pdl);
     case EPI_QKV: return launch_t<BN, EPI_QKV>(ma, mb, kp, st, pdl);
+    case EPI_LSE: return launch_t<BN, EPI_LSE>(ma, mb, kp, st, pdl);
   }
   return cudaErrorInvalidValue;
 }
 
+__global__ void lse_combine_kernel(const float2* part, int ld, int m_tiles, int T, float* lse) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= T) return;
+  float mx = -INFINITY;
+  for (int m = 0; m < m_tiles; ++m) mx = fmaxf(mx, part[(size_t)m * ld + t].x);
+  float s = 0.f;
+  if (mx != -INFINITY)
+    for (int m = 0; m < m_tiles; ++m) {
+      const float2 v = part[(size_t)m * ld + t];
+      if (v.x != -INFINITY) s += v.y * expf(v.x - mx);
+    }
+  lse[t] = mx + logf(s);
+}
+
 }  // namespace
+
+cudaError_t lse_combine_launch(const float2* part, int ld, int m_tiles, int T, float* lse, cudaStream_t st) {
+  if (T <= 0) return cudaSuccess;
+  lse_combine_kernel<<<(T + 127) / 128, 128, 0, st>>>(part, ld, m_tiles, T, lse);
+  return cudaGetLastError();
+}
 
 bool gemm_make_map(CUtensorMap* m, const void* base, int inner, int rows, int box_rows, char* eb, size_t el) {
   return make_map(m, base, inner, rows, box_rows, eb, el);

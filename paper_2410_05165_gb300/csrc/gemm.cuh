@@ -8,7 +8,7 @@
 
 namespace atspeed {
 
-enum EpiKind : int { EPI_F32 = 0, EPI_BF16 = 1, EPI_RESID = 2, EPI_SWIGLU = 3, EPI_QKV = 4 };
+enum EpiKind : int { EPI_F32 = 0, EPI_BF16 = 1, EPI_RESID = 2, EPI_SWIGLU = 3, EPI_QKV = 4, EPI_LSE = 5 };
 
 // Y[t][m] = sum_k W[m][k] * X[t][k]  (W: weight rows, X: token rows, both bf16 K-major)
 // with a fused epilogue.  The MMA runs "swap-AB": weight rows are the MMA M dimension (128 per
@@ -26,6 +26,10 @@ struct GemmArgs {
   float* out_f32;           // EPI_F32 / EPI_RESID: [T][ldo]
   __nv_bfloat16* out_bf16;  // EPI_BF16 / EPI_SWIGLU: [T][ldo]
   int ldo;
+  // EPI_LSE: per (weight-row tile, token) the tile's (max, sum of exp(y - max)) over its rows,
+  // lse_part[m_tile * lse_ld + token] (the logits themselves are not stored)
+  float2* lse_part;
+  int lse_ld;
   // EPI_QKV
   int d_model, head_dim;
   const int* pos;           // [T] rotary positions
@@ -44,6 +48,10 @@ struct GemmScratch {
   int max_tiles;
   unsigned int* err;        // device error word
 };
+
+// log-sum-exp of each token's whole row from the EPI_LSE partials of m_tiles row tiles, combined in
+// tile order: lse[t] = log sum_m s_m exp(max_m - max) + max.
+cudaError_t lse_combine_launch(const float2* part, int ld, int m_tiles, int T, float* lse, cudaStream_t st);
 
 // Bytes of split-K workspace / counters needed for a grid of `grid` CTAs.
 size_t gemm_ws_bytes(int grid);

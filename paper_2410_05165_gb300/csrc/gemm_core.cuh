@@ -192,6 +192,36 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, in
         out[(size_t)tok * a.ldo] = __float2bfloat16_rn(g / (1.0f + expf(-g)) * u);
       }
     }
+  } else if constexpr (EPI == EPI_LSE) {
+    // per token of the chunk, (max, sum of exp(y - max)) over the tile's rows: 4 threads per token
+    // take 32 rows each (rotated by token and thread so the shared-memory reads spread over the
+    // banks), then combine in a fixed order (pairs, then pairs of pairs)
+    const int j = ep_tid >> 2, sub = ep_tid & 3;
+    const int valid = min(GEMM_BM, a.M - m_tile * GEMM_BM);
+    const float* sj = st + j * GEMM_BM + sub * 32;
+    float mx = -INFINITY;
+#pragma unroll 8
+    for (int i = 0; i < 32; ++i) {
+      const int r = (i + sub * 8 + j) & 31;
+      if (sub * 32 + r < valid) mx = fmaxf(mx, sj[r]);
+    }
+    float sm = 0.f;
+    if (mx != -INFINITY) {
+#pragma unroll 8
+      for (int i = 0; i < 32; ++i) {
+        const int r = (i + sub * 8 + j) & 31;
+        if (sub * 32 + r < valid) sm += expf(sj[r] - mx);
+      }
+    }
+#pragma unroll
+    for (int o = 1; o <= 2; o <<= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, mx, o), s2 = __shfl_xor_sync(0xffffffffu, sm, o);
+      const float mn = fmaxf(mx, m2);
+      sm = (mx == -INFINITY ? 0.f : sm * expf(mx - mn)) + (m2 == -INFINITY ? 0.f : s2 * expf(m2 - mn));
+      mx = mn;
+    }
+    const int tok = tok0 + j;
+    if (sub == 0 && tok < a.T) a.lse_part[(size_t)m_tile * a.lse_ld + tok] = make_float2(mx, sm);
   } else {
     // thread owns weight row m of the tile and the 32 tokens of the chunk
     const int m = ep_tid;

@@ -235,25 +235,31 @@ __device__ __forceinline__ int trie_child(const TreeDev& t, int x, int c) {
   return t.trie_child[x] + r;
 }
 
-// One warp: MASKED constrained log-probs of the valid children of trie node `tn`, given the 256
-// logits of the node's level.  Lane l owns codes 8l .. 8l+7; returns the valid bits of those codes.
-__device__ __forceinline__ uint32_t warp_logprobs(const float* row, const uint32_t* tmask, int tn, float (&lp)[8]) {
+// One warp: constrained log-probs of the valid children of trie node `tn`, given the 256 logits of
+// the node's level: MASKED (log-sum-exp over the valid children) when lse_full is NaN, else FULL
+// (lse_full = log-sum-exp of the node's whole-vocabulary row).  Lane l owns codes 8l .. 8l+7;
+// returns the valid bits of those codes.
+__device__ __forceinline__ uint32_t warp_logprobs(const float* row, const uint32_t* tmask, int tn, float (&lp)[8],
+                                                  float lse_full) {
   const int lane = threadIdx.x & 31;
   const uint32_t bits = (tmask[(size_t)tn * 8 + (lane >> 2)] >> ((lane & 3) * 8)) & 0xFFu;
   const float4 x0 = *reinterpret_cast<const float4*>(row + lane * 8);
   const float4 x1 = *reinterpret_cast<const float4*>(row + lane * 8 + 4);
   const float x[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-  float m = -INFINITY;
+  float lse = lse_full;
+  if (isnan(lse_full)) {
+    float m = -INFINITY;
 #pragma unroll
-  for (int j = 0; j < 8; ++j)
-    if (bits >> j & 1u) m = fmaxf(m, x[j]);
-  m = warp_max(m);
-  float s = 0.f;
+    for (int j = 0; j < 8; ++j)
+      if (bits >> j & 1u) m = fmaxf(m, x[j]);
+    m = warp_max(m);
+    float s = 0.f;
 #pragma unroll
-  for (int j = 0; j < 8; ++j)
-    if (bits >> j & 1u) s += expf(x[j] - m);
-  s = warp_sum(s);
-  const float lse = m + logf(s);
+    for (int j = 0; j < 8; ++j)
+      if (bits >> j & 1u) s += expf(x[j] - m);
+    s = warp_sum(s);
+    lse = m + logf(s);
+  }
 #pragma unroll
   for (int j = 0; j < 8; ++j) lp[j] = x[j] - lse;
   return bits;
@@ -298,7 +304,7 @@ __global__ void __launch_bounds__(NT) draft_level_kernel(TreeDev t, int lvl, int
     const size_t node = base + poff + p;
     const float* row = t.logits_d + (size_t)t.lg_d[node] * ITEM_ROWS + (d + lvl - 1) * TREE_CODES;
     float lp[8];
-    const uint32_t bits = warp_logprobs(row, t.trie_mask, t.trie[node], lp);
+    const uint32_t bits = warp_logprobs(row, t.trie_mask, t.trie[node], lp, t.lse_d ? t.lse_d[t.lg_d[node]] : NAN);
     const float sq0 = t.sq[node];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
@@ -379,7 +385,7 @@ __global__ void __launch_bounds__(NT) verify_strict_kernel(TreeDev t, int K, Ver
       const int node = yp_node[p];
       const float* row = t.logits_t + (size_t)t.lg_t[node] * ITEM_ROWS + (d + j - 1) * TREE_CODES;
       float lp[8];
-      const uint32_t bits = warp_logprobs(row, t.trie_mask, t.trie[node], lp);
+      const uint32_t bits = warp_logprobs(row, t.trie_mask, t.trie[node], lp, t.lse_t ? t.lse_t[t.lg_t[node]] : NAN);
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
         const int idx = p * TREE_CODES + lane * 8 + q;
@@ -492,14 +498,14 @@ __global__ void __launch_bounds__(NT) verify_relaxed_kernel(TreeDev t, int K, Ve
       const size_t node = base + poff + p;
       const float* rp = t.logits_t + (size_t)t.lg_t[node] * ITEM_ROWS + (lvl_abs - 1) * TREE_CODES;
       float lp[8];
-      const uint32_t bits = warp_logprobs(rp, t.trie_mask, t.trie[node], lp);
+      const uint32_t bits = warp_logprobs(rp, t.trie_mask, t.trie[node], lp, t.lse_t ? t.lse_t[t.lg_t[node]] : NAN);
       const float spn = t.sp[node];
 #pragma unroll
       for (int q = 0; q < 8; ++q) Sp[p * TREE_CODES + lane * 8 + q] = (bits >> q & 1u) ? spn + lp[q] : -INFINITY;
       if (j <= g) {
         const float* rq = t.logits_d + (size_t)t.lg_d[node] * ITEM_ROWS + (lvl_abs - 1) * TREE_CODES;
         float lq[8];
-        warp_logprobs(rq, t.trie_mask, t.trie[node], lq);
+        warp_logprobs(rq, t.trie_mask, t.trie[node], lq, t.lse_d ? t.lse_d[t.lg_d[node]] : NAN);
         const float sqn = (plvl == 0) ? spn : t.sq[node];
 #pragma unroll
         for (int q = 0; q < 8; ++q) Sq[p * TREE_CODES + lane * 8 + q] = (bits >> q & 1u) ? sqn + lq[q] : -INFINITY;

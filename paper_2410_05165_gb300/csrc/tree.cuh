@@ -39,6 +39,10 @@ struct TreeDev {
   // item-code logits [rows][1024]: block l*256 .. l*256+255 scores the codes of level l
   const float* logits_t;
   const float* logits_d;
+  // FULL normalisation: log-sum-exp of each logits row's whole-vocabulary row (same row index as
+  // logits_t / logits_d); null under MASKED normalisation
+  const float* lse_t;
+  const float* lse_d;
 };
 
 __host__ __device__ inline int level_off(const TreeDev& t, int lvl) {

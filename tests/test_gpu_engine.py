@@ -314,3 +314,108 @@ def test_persistent_forward_equals_per_op_multi_user(ats, cfg, layers, B, monkey
         ctx.close()
     assert np.all(np.isfinite(outs[0]))
     np.testing.assert_array_equal(outs[0], outs[1])
+
+
+# ------------------------------------------------------------------------------------------------
+# FULL normalisation (whole-vocabulary log-softmax, then the trie mask)
+# ------------------------------------------------------------------------------------------------
+
+def _near_tie_level(item_rows, full_rows, trie, K, tol):
+    """Whether the oracle's FULL plain beam search meets, at some level, K-th and (K+1)-th
+    candidates closer than tol."""
+    from oracle.beam import child_paths, expand, topk
+    beams, sp = [()], np.zeros(1, np.float32)
+    for _ in range(L):
+        C = expand(beams, sp, item_rows(beams), trie, full_rows(beams))
+        sc = np.sort(C.score.astype(np.float64))[::-1]
+        if sc.size > K and sc[K - 1] - sc[K] < tol:
+            return True
+        sel = topk(C, K)
+        beams, sp = child_paths(beams, C, sel), C.score[sel]
+    return False
+
+
+@pytest.mark.parametrize("cfg,layers", [("tiny", None), ("mid", 2)])
+def test_full_norm_node_lse_matches_oracle(ats, cfg, layers):
+    """Whole-vocabulary log-sum-exp of the prefill row and of every node of a seeded drafted tree
+    (the LM head over all V rows with the log-sum-exp epilogue) against logsumexp of the oracle's
+    whole-vocabulary logits of prompt + path."""
+    import scipy.special
+    w = synth.workload(cfg)
+    spec = w.target if layers is None else synth.ModelSpec(layers, w.target.d_model, w.target.n_heads,
+                                                          w.target.d_ffn, w.target.vocab)
+    items = synth.make_items(min(w.n_items, 5000), w.code_dist, w.zipf_a, w.seed)
+    prompt = synth.make_prompts(1, w.prompt_len, spec.vocab, w.seed)[0]
+    K, N, G = w.K, w.N, 3
+    ctx = _ctx(ats, spec, None, items, w.code_base, 1, len(prompt), K, N, G, seed=w.seed)
+    _prefill(ats, ctx, [prompt])
+    incoming, levels = synth.random_tree(items, 0, 1, G, N, seed=5)
+    o = ats.opts(K, N, G, norm=ats.NORM_FULL)
+    ctx.begin_step(o)
+    cnt, par, cod, sq = _tree_arrays(levels, 1, G, N)
+    ctx.set_tree(cnt, par, cod, sq)
+    ctx.verify(o, ats.STRICT)
+    ev = PathEvaluator(Model(spec, synth.model_weights(spec, w.seed, "target"), w.code_base), prompt,
+                       full_vocab=True)
+    errs = [abs(ctx.node_lse(0, 0, 0) - float(scipy.special.logsumexp(ev.root_logits)))]
+    off, prev = K, [()]
+    for lvl in levels:
+        cur = [prev[p] + (c,) for p, c in lvl]
+        for k, row in enumerate(ev.logits(cur)):
+            errs.append(abs(ctx.node_lse(0, 0, off + k) - float(scipy.special.logsumexp(row))))
+        off += N
+        prev = cur
+    errs = np.array(errs)
+    print(f"{cfg}: |lse - oracle| max {errs.max():.3g} mean {errs.mean():.3g} over {errs.size} rows")
+    # the log-sum-exp moves by at most the largest logit error: the node-logit bounds apply
+    assert errs.mean() < 2e-2 and errs.max() < 0.1, (errs.mean(), errs.max())
+    ctx.close()
+
+
+def test_full_norm_sd_lossless_and_matches_oracle_tiny(ats):
+    """FULL normalisation end to end on the tiny workload: strict SD == plain target beam search
+    bit for bit on the GPU, equal to the oracle's FULL plain beam search up to near-ties; relaxed
+    SD returns K distinct valid items ranked by score."""
+    import scipy.special
+    w = synth.workload("tiny")
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    prompts = synth.make_prompts(2, w.prompt_len, w.target.vocab, w.seed)
+    ctx = _ctx(ats, w.target, w.draft, items, w.code_base, 2, 32, w.K, w.N, w.gamma, seed=w.seed)
+    toks = torch.from_numpy(np.concatenate(prompts)).cuda()
+    off = [0, len(prompts[0]), len(prompts[0]) + len(prompts[1])]
+    o = ats.opts(w.K, w.N, w.gamma, norm=ats.NORM_FULL)
+    sd_items, sd_sc, stats = ctx.beam_search(toks, off, o, ats.SD_STRICT)
+    pl_items, pl_sc, _ = ctx.beam_search(toks, off, o, ats.PLAIN_TOPK)
+    np.testing.assert_array_equal(sd_items.cpu().numpy(), pl_items.cpu().numpy())
+    np.testing.assert_array_equal(sd_sc.cpu().numpy(), pl_sc.cpu().numpy())
+    m_items, m_sc, _ = ctx.beam_search(toks, off, ats.opts(w.K, w.N, w.gamma), ats.PLAIN_TOPK)
+    assert not np.array_equal(m_sc.cpu().numpy(), pl_sc.cpu().numpy())   # the two normalisations differ
+    tw = synth.model_weights(w.target, w.seed, "target")
+    trie = Trie(items)
+    cb = w.code_base
+    tol = 4 * 2e-2   # L = 4 log-probs per score, each within 2e-2
+    for u in range(2):
+        ev = PathEvaluator(Model(w.target, tw, cb), prompts[u], full_vocab=True)
+        item_rows = lambda ps: [ev.logits([p])[0][cb + 256 * len(p):cb + 256 * (len(p) + 1)].astype(np.float32)
+                                for p in ps]
+        full_rows = lambda ps: [ev.logits([p])[0].astype(np.float32) for p in ps]
+        ref, ref_sc = plain_beam_search(item_rows, trie, w.K, full_rows=full_rows)
+        got = [tuple(int(c) for c in r) for r in sd_items[u].cpu().numpy()]
+        # every returned item's score is the oracle's FULL score of that item
+        for it, sc in zip(got, sd_sc[u].cpu().numpy()):
+            ref_item = sum(float(r[cb + 256 * l + it[l]]) - float(scipy.special.logsumexp(r.astype(np.float64)))
+                           for l, r in enumerate(full_rows([it[:l] for l in range(4)])))
+            assert abs(float(sc) - ref_item) < tol, (it, sc, ref_item)
+        # the lists agree unless a level's K-th and (K+1)-th candidates are within the score bound
+        # (the GPU may then keep the other beam, and every later level differs)
+        if got != ref:
+            assert _near_tie_level(item_rows, full_rows, trie, w.K, tol), (got, ref)
+        else:
+            np.testing.assert_allclose(sd_sc[u].cpu().numpy(), ref_sc, atol=tol)
+    rx_items, rx_sc, _ = ctx.beam_search(toks, off, o, ats.SD_RELAXED)
+    valid = {tuple(int(c) for c in it) for it in items}
+    for u in range(2):
+        got = [tuple(int(c) for c in r) for r in rx_items[u].cpu().numpy()]
+        assert len(set(got)) == w.K and all(g in valid for g in got)
+        assert np.all(np.diff(rx_sc[u].cpu().numpy()) <= 0)
+    ctx.close()

@@ -102,10 +102,12 @@ def test_7b_relaxed_outputs_are_valid_distinct_ranked(ats, world):
     ctx.close()
 
 
-@pytest.mark.parametrize("B,K,gamma,N", [(4, 5, 2, 10), (1, 20, 3, 80), (4, 1, 4, 4)])
-def test_7b_sweep_points_strict_lossless(ats, world, B, K, gamma, N):
-    """Points of the verification-call sweep (batch x K x gamma x N, 512-token histories): strict
-    speculative decoding returns the plain target beam search's lists bit for bit, for every user."""
+@pytest.mark.parametrize("B,K,gamma,N,full", [(4, 5, 2, 10, False), (1, 20, 3, 80, False), (4, 1, 4, 4, False),
+                                               (1, 10, 4, 40, True)])
+def test_7b_sweep_points_strict_lossless(ats, world, B, K, gamma, N, full):
+    """Points of the verification-call sweep (batch x K x gamma x N, 512-token histories), and the
+    bench point under FULL normalisation: strict speculative decoding returns the plain target beam
+    search's lists bit for bit, for every user."""
     w, _, _, items, _, _ = world
     prompts = synth.make_prompts(B, w.prompt_len, w.target.vocab, w.seed + 7)
     P = [len(p) for p in prompts]
@@ -113,7 +115,7 @@ def test_7b_sweep_points_strict_lossless(ats, world, B, K, gamma, N):
                       max_K=20, max_N=80, max_gamma=4)
     toks = torch.from_numpy(np.concatenate(prompts).astype(np.int32)).cuda()
     off = np.concatenate([[0], np.cumsum(P)]).astype(np.int32).tolist()
-    o = ats.opts(K, N, gamma, w.philox_seed)
+    o = ats.opts(K, N, gamma, w.philox_seed, norm=ats.NORM_FULL if full else ats.NORM_MASKED)
     sd_items, sd_sc, stats = ctx.beam_search(toks, off, o, ats.SD_STRICT)
     pl_items, pl_sc, _ = ctx.beam_search(toks, off, o, ats.PLAIN_TOPK)
     np.testing.assert_array_equal(sd_items.cpu().numpy(), pl_items.cpu().numpy())
