@@ -80,6 +80,10 @@ def parse():
                          "K in {1,5,10,20} x gamma in {1..4} x N in {K,2K,4K} x batch in {1,4,16}, strict and "
                          "relaxed; one JSON line per point")
     ap.add_argument("--sweep-batches", default="1,4,16", help="--sweep: the batch axis")
+    ap.add_argument("--tree-vs-beam", action="store_true",
+                    help="one target decoding step of beam width W: the W beams as one tree sharing the "
+                         "user's history (tree attention) against W separate sequences, each with its own "
+                         "copy of the history; one JSON line per W")
     return ap.parse_args()
 
 
@@ -491,9 +495,59 @@ def sweep(batches, reps=2):
         ctx.close()
 
 
+def tree_vs_beam(widths=(5, 10, 20, 40, 80), reps=3):
+    """Cost of one target decoding step of beam search with W beams at depth 1 of the item (the
+    analogue of the paper's tree-attention speedup, Sec. 4 / appendix): the W beams forwarded as
+    one tree whose nodes share the user's 512-token history in the paged KV cache, against W
+    independent sequences, each prefilled with its own copy of the history (W users of one beam).
+    Both calls forward W tokens through the 7B-shape target; the first reads one history's K/V
+    per layer, the second W of them."""
+    import torch
+    import paper_2410_05165_gb300 as ats
+    ats.load()
+    w = synth.workload("7b")
+    tw = {n: torch.from_numpy(a).to(device="cuda", dtype=torch.bfloat16)
+          for n, a in synth.iter_model_tensors(w.target, w.seed, "target")}
+    dw = {n: torch.from_numpy(a).to(device="cuda", dtype=torch.bfloat16)
+          for n, a in synth.iter_model_tensors(w.draft, w.seed, "draft")}
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    prompt = synth.make_prompts(1, w.prompt_len, w.target.vocab, w.seed)[0]
+
+    def call_ms(B, K):
+        ctx = ats.Context(w.target, tw, w.draft, dw, items, w.code_base, max_users=B, max_prompt=len(prompt),
+                          max_K=K, max_N=K, max_gamma=1)
+        toks = torch.from_numpy(np.concatenate([prompt] * B).astype(np.int32)).cuda()
+        off = (np.arange(B + 1) * len(prompt)).astype(np.int32)
+        o = ats.opts(K, K, 1, w.philox_seed)
+        ms, T = [], 0
+        for _ in range(reps):
+            ctx.prefill(toks, off)
+            ctx.begin_step(o)
+            ctx.draft_step(o, ats.STRICT)
+            T = int(ctx.debug_tree(1)["count"][:, 1].sum())
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            ctx.verify(o, ats.STRICT)
+            e1.record()
+            torch.cuda.synchronize()
+            ms.append(e0.elapsed_time(e1))
+        ctx.close()
+        return float(np.median(ms)), T
+
+    for W in widths:
+        tree_ms, tree_T = call_ms(1, W)
+        beam_ms, beam_T = call_ms(W, 1)
+        print(json.dumps({"tree_vs_beam": W, "tree_tokens": tree_T, "tree_ms": round(tree_ms, 4),
+                          "per_beam_tokens": beam_T, "per_beam_ms": round(beam_ms, 4),
+                          "speedup": round(beam_ms / tree_ms, 3)}), flush=True)
+
+
 def main():
     args = parse()
     w = synth.workload(args.workload)
+    if args.tree_vs_beam:
+        tree_vs_beam()
+        return
     if args.sweep:
         sweep([int(b) for b in args.sweep_batches.split(",")])
         return
