@@ -67,7 +67,8 @@ struct ModelRt {
   // per-token forward inputs
   int *tok = nullptr, *pos = nullptr, *kvrow = nullptr, *tuser = nullptr, *tvis = nullptr, *anc = nullptr,
       *ancn = nullptr;
-  int *qt_t0 = nullptr, *qt_n = nullptr, *qt_user = nullptr, *rows_sel = nullptr, *user_splits = nullptr;
+  int *qt_t0 = nullptr, *qt_n = nullptr, *qt_user = nullptr, *qt_vis = nullptr, *rows_sel = nullptr,
+      *user_splits = nullptr;
   float *part_o = nullptr, *part_ml = nullptr;
   int max_splits = 1;
   // persistent forward kernel
@@ -318,6 +319,7 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.qt_t0 = dalloc<int>(c, max_qt);
   m.qt_n = dalloc<int>(c, max_qt);
   m.qt_user = dalloc<int>(c, max_qt);
+  m.qt_vis = dalloc<int>(c, max_qt);
   m.rows_sel = dalloc<int>(c, m.Tcap);
   m.user_splits = dalloc<int>(c, L.max_users);
   const int pages = c->prefix_pages_per_user;
@@ -468,7 +470,7 @@ struct FwdPlan {
   int T = 0;
   bool prefill = false;
   const int* d_tokens = nullptr;       // prefill: caller's tokens; tree: m.tok (filled by gather)
-  std::vector<int> qt_t0, qt_n, qt_user;
+  std::vector<int> qt_t0, qt_n, qt_user, qt_vis;   // qt_vis: longest visible prefix in the tile
   std::vector<int> splits;             // per user
   std::vector<int> out_rows;           // tokens whose logits are produced, in order
   int logit_row_base = 0;
@@ -532,6 +534,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
   CK(cudaMemcpyAsync(m.qt_t0, p.qt_t0.data(), nqt * 4, cudaMemcpyHostToDevice, st));
   CK(cudaMemcpyAsync(m.qt_n, p.qt_n.data(), nqt * 4, cudaMemcpyHostToDevice, st));
   CK(cudaMemcpyAsync(m.qt_user, p.qt_user.data(), nqt * 4, cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(m.qt_vis, p.qt_vis.data(), nqt * 4, cudaMemcpyHostToDevice, st));
   CK(cudaMemcpyAsync(m.user_splits, p.splits.data(), p.splits.size() * 4, cudaMemcpyHostToDevice, st));
   CK(cudaMemcpyAsync(m.rows_sel, p.out_rows.data(), p.out_rows.size() * 4, cudaMemcpyHostToDevice, st));
   int max_split = 1;
@@ -585,6 +588,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     a.qt_t0 = m.qt_t0;
     a.qt_n = m.qt_n;
     a.qt_user = m.qt_user;
+    a.qt_vis = m.qt_vis;
     a.tok_user = m.tuser;
     a.tok_vis = m.tvis;
     a.anc_row = p.prefill ? nullptr : m.anc;
@@ -652,6 +656,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     a.qt_t0 = m.qt_t0;
     a.qt_n = m.qt_n;
     a.qt_user = m.qt_user;
+    a.qt_vis = m.qt_vis;
     a.tok_user = m.tuser;
     a.tok_vis = m.tvis;
     a.anc_row = p.prefill ? nullptr : m.anc;
@@ -748,11 +753,15 @@ void full_lse(atspeed_ctx* c, ModelRt& m, const bf16* X, int X_rows, int n, floa
   c->n_launch += 1;
 }
 
-void add_qtiles(FwdPlan& p, int u, int t0, int n) {
+// Query tiles of user u's n consecutive tokens from t0.  vis = the history length every token sees
+// (tree nodes), or -1 for the history itself (token i sees i + 1 tokens).
+void add_qtiles(FwdPlan& p, int u, int t0, int n, int vis) {
   for (int i = 0; i < n; i += ATT_QTILE) {
+    const int cnt = std::min(ATT_QTILE, n - i);
     p.qt_t0.push_back(t0 + i);
-    p.qt_n.push_back(std::min(ATT_QTILE, n - i));
+    p.qt_n.push_back(cnt);
     p.qt_user.push_back(u);
+    p.qt_vis.push_back(vis < 0 ? i + cnt : vis);
   }
 }
 
@@ -781,7 +790,7 @@ void forward_nodes(atspeed_ctx* c, ModelRt& m, bool target, const std::vector<in
     const int u = nodes[i] / t.stride;
     int j = i;
     while (j < T && nodes[j] / t.stride == u) ++j;
-    add_qtiles(p, u, i, j - i);
+    add_qtiles(p, u, i, j - i, c->users[u].P);
     i = j;
   }
   p.splits.resize(c->B);
@@ -1087,7 +1096,7 @@ void prefill_impl(atspeed_ctx* c, cudaStream_t st, int n_users, const int32_t* d
       tuser[t0 + i] = u;
       tvis[t0 + i] = i + 1;
     }
-    add_qtiles(p, u, t0, P[u]);
+    add_qtiles(p, u, t0, P[u], -1);
     p.out_rows.push_back(t0 + P[u] - 1);
     UserState& us = c->users[u];
     us.P = P[u];

@@ -21,7 +21,6 @@ __global__ void __launch_bounds__(128)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::SMEM_BODY);
-  int* s_info = reinterpret_cast<int*>(bars + 2);
   pdl_launch_dependents();
   pdl_wait();
   if (threadIdx.x == 0) {
@@ -33,7 +32,7 @@ __global__ void __launch_bounds__(128)
   }
   __syncthreads();
   int use[2] = {0, 0};
-  attn_item<HD>(a, &mk, &mv, blockIdx.x, blockIdx.y, blockIdx.z, smem, bars, s_info, use, threadIdx.x, 1);
+  attn_item<HD>(a, &mk, &mv, blockIdx.x, blockIdx.y, blockIdx.z, smem, bars, use, threadIdx.x, 1);
 }
 
 // One CTA of 128 threads per (query tile, head, group of 16 queries): merge the prefix splits with

@@ -29,6 +29,7 @@ struct AttnArgs {
   const int* qt_t0;                // [n_qtiles] first token of the tile
   const int* qt_n;                 // [n_qtiles] tokens in the tile (<= 64)
   const int* qt_user;              // [n_qtiles]
+  const int* qt_vis;               // [n_qtiles] longest visible prefix of the tile's tokens
   // per token
   const int* tok_user;             // [T] user of each token
   const int* tok_vis;              // [T] visible prefix length (P for tree nodes, pos+1 for prefill)

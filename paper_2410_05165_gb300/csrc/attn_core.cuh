@@ -79,7 +79,7 @@ struct AttCfg {
 // a bounded wait timed out.
 template <int HD>
 __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtensorMap* mv, int tile, int h, int split,
-                          uint8_t* smem, uint64_t* bars, int* s_info, int (&use)[2], int tid, int bar_id,
+                          uint8_t* smem, uint64_t* bars, int (&use)[2], int tid, int bar_id,
                           unsigned long long* tr = nullptr, size_t trs = 0) {
 #define ATT_TR(k) do { if (tr && tid == 0) tr[(size_t)(k) * trs] = globaltimer_ns(); } while (0)
   using C = AttCfg<HD>;
@@ -95,21 +95,17 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
   const int S_u = a.user_splits[u];
   if (split >= S_u) return true;
 
-  // longest visible prefix of the tile's queries (one load per thread, then a max over the CTA)
-  {
-    int mv_ = 0;
-    if (tid < nq) mv_ = a.tok_vis[t0 + tid];
-    if (tid + 128 < nq) mv_ = max(mv_, a.tok_vis[t0 + tid + 128]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mv_ = max(mv_, __shfl_xor_sync(0xffffffffu, mv_, o));
-    if (lane == 0) s_info[2 + warp] = mv_;
-  }
-  named_bar_sync(bar_id, 128);
-  ATT_TR(0);
+  // this item's prefix pages [c0, c1): the split's share of the pages the tile's queries see
   const int* ptab = a.page_table + (size_t)u * a.max_pages;
   constexpr int NBOX = HD >= 64 ? HD / 64 : 1;
   constexpr int BOXW = HD >= 64 ? 64 : HD;
-  int c0 = 0, c1 = 0;   // this item's prefix pages: thread 0 computes them, the others read s_info
+  const int nch = (a.qt_vis[tile] + ATT_PAGE - 1) / ATT_PAGE;
+  int c0 = 0, c1 = nch;
+  if (a.chunks_per_split > 0) {
+    c0 = min(nch, split * a.chunks_per_split);
+    c1 = min(nch, c0 + a.chunks_per_split);
+  }
+  ATT_TR(0);
   int page0 = 0, page1 = 0;   // cache pages of the first two pages (thread 0)
   // copy of half page sc (keys sc * ATT_SUB ...) into buffer buf
   auto issue = [&](int sc, int buf) {
@@ -124,22 +120,11 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
     }
   };
   constexpr int SUBS = ATT_PAGE / ATT_SUB;
-  if (tid == 0) {
-    const int mv_ = max(max(s_info[2], s_info[3]), max(s_info[4], s_info[5]));
-    const int nch = (mv_ + ATT_PAGE - 1) / ATT_PAGE;
-    c1 = nch;
-    if (a.chunks_per_split > 0) {
-      c0 = min(nch, split * a.chunks_per_split);
-      c1 = min(nch, c0 + a.chunks_per_split);
-    }
-    s_info[0] = c0;
-    s_info[1] = c1;
-    // the first K / V half page does not depend on Q: start its copy now
-    if (c0 < c1) {
-      page0 = ptab[c0];
-      if (c0 + 1 < c1) page1 = ptab[c0 + 1];
-      issue(c0 * SUBS, 0);
-    }
+  // the first K / V half page does not depend on Q: start its copy now
+  if (tid == 0 && c0 < c1) {
+    page0 = ptab[c0];
+    if (c0 + 1 < c1) page1 = ptab[c0 + 1];
+    issue(c0 * SUBS, 0);
   }
   // Q tile -> shared memory (rows >= nq are zero); all of a thread's loads are issued first
   {
@@ -161,8 +146,6 @@ __device__ bool attn_item(const AttnArgs& a, const CUtensorMap* mk, const CUtens
   }
   named_bar_sync(bar_id, 128);
   ATT_TR(1);
-  c0 = s_info[0];
-  c1 = s_info[1];
 
   // Q fragments (A operand) for this warp's 16 rows
   uint32_t qf[NKS][4];

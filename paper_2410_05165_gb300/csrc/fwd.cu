@@ -447,7 +447,7 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
 // prefix split) are item c + (2k + wg) G; each is followed by the warpgroup's share of the merge of
 // the splits of (tile, head) once all of them are published.
 template <int HD>
-__device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* att_smem, uint64_t* att_bars, int* s_info,
+__device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* att_smem, uint64_t* att_bars,
                                            int (&use_att)[2], int* flag, int wt, int wg, int wbar) {
   const int c = blockIdx.x, G = p.G, L = p.L;
   AttnArgs a = p.att_args;
@@ -463,7 +463,7 @@ __device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* a
     const int h = rem / S, split = rem % S;
     const bool tr_on = p.trace && wg == 0 && nit == 0;
     unsigned long long* tr = tr_on ? p.trace + ((size_t)8 * NP + ph) * G + c : nullptr;
-    if (!attn_item<HD>(a, mk, mv, tile, h, split, att_smem, att_bars, s_info, use_att, wt, wbar, tr, (size_t)NP * G))
+    if (!attn_item<HD>(a, mk, mv, tile, h, split, att_smem, att_bars, use_att, wt, wbar, tr, (size_t)NP * G))
       return false;
     if (tr_on && wt == 0) p.trace[((size_t)4 * NP + ph) * G + c] = globaltimer_ns();
     if (a.direct) continue;
@@ -721,8 +721,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
   int* go = failed + 1;   // count of GEMM phases whose input the compute warps have seen published
   int* lastA = go + 1;                                            // [SA] parity of last fill, -1 none
   int* lastB = lastA + C::SA;                                     // [SB]
-  int* s_info = lastB + C::SB;                                    // 6 per warpgroup (attention)
-  float* red = reinterpret_cast<float*>(s_info + 12);             // 8
+  float* red = reinterpret_cast<float*>(lastB + C::SB);           // 8
   int* part_slot = reinterpret_cast<int*>(red + 8);               // 256
   int* tpos = part_slot + 256;                                    // [BN] QKV token tables
   int* tkvr = tpos + 256;
@@ -730,7 +729,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
   int* tslot = toff + 68;                                         // [PART_TABLE_CAP]
   GemmArgs* s_ea = reinterpret_cast<GemmArgs*>((reinterpret_cast<uintptr_t>(tslot + PART_TABLE_CAP) + 15) &
                                                 ~uintptr_t(15));   // epilogue arguments
-  static_assert(8 * (2 * C::SA + 2 * C::SB + 9) + 4 * (6 + C::SA + C::SB + 12 + 8 + 256 + 512 + 68 + PART_TABLE_CAP) + 16 + (int)sizeof(GemmArgs) <=
+  static_assert(8 * (2 * C::SA + 2 * C::SB + 9) + 4 * (6 + C::SA + C::SB + 8 + 256 + 512 + 68 + PART_TABLE_CAP) + 16 + (int)sizeof(GemmArgs) <=
                     C::MISC,
                 "shared-memory misc area too small");
 
@@ -964,7 +963,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
         norm_phase<BN>(p, nmode, ng, red, rowbuf, ctid, 4 * l + (kind == 3 ? 1 : 3), toff, tslot, tab_nt, ph);
       } else if (kind == 2) {
         // both warpgroups leave together: a failed bounded wait in either ends the program
-        const bool aok = attn_phase<HD>(p, l, att_smem + wg * LY::ATT_BODY, att_bars + 2 * wg, s_info + 6 * wg,
+        const bool aok = attn_phase<HD>(p, l, att_smem + wg * LY::ATT_BODY, att_bars + 2 * wg,
                                         use_att, flagw + wg, wt, wg, 2 + wg);
         if (!named_bar_and(1, CT, aok)) {
           ok = false;

@@ -110,7 +110,7 @@ size_t atspeed_op_attention_scratch(int T, int n_heads, int head_dim, int P) {
   const int S = std::max(1, (pages + 1) / 2);
   const int nqt = (T + ATT_QTILE - 1) / ATT_QTILE;
   const size_t floats = (size_t)S * T * n_heads * head_dim + (size_t)S * T * n_heads * 2;
-  const size_t ints = (size_t)3 * nqt + (size_t)T * 7 + pages + 1;
+  const size_t ints = (size_t)4 * nqt + (size_t)T * 7 + pages + 1;
   return floats * 4 + ints * 4 + 256;
 }
 
@@ -138,7 +138,7 @@ atspeed_status atspeed_op_attention(atspeed_stream stream, const void* d_q, cons
   float* part_o = static_cast<float*>(d_part);
   float* part_ml = part_o + (size_t)S * T * n_heads * head_dim;
   int* ip = reinterpret_cast<int*>(part_ml + (size_t)S * T * n_heads * 2);
-  std::vector<int> host(3 * nqt + 7 * T + pages + 1, 0);
+  std::vector<int> host(4 * nqt + 7 * T + pages + 1, 0);
   int* qt0 = host.data();
   int* qtn = qt0 + nqt;
   int* qtu = qtn + nqt;
@@ -148,6 +148,7 @@ atspeed_status atspeed_op_attention(atspeed_stream stream, const void* d_q, cons
   int* ann = an + 4 * T;
   int* pg = ann + T;
   int* sp = pg + pages;
+  int* qtv = sp + 1;
   for (int i = 0; i < nqt; ++i) {
     qt0[i] = i * ATT_QTILE;
     qtn[i] = std::min(ATT_QTILE, T - i * ATT_QTILE);
@@ -155,6 +156,7 @@ atspeed_status atspeed_op_attention(atspeed_stream stream, const void* d_q, cons
   }
   for (int t = 0; t < T; ++t) {
     tv[t] = h_vis[t];
+    qtv[t / ATT_QTILE] = std::max(qtv[t / ATT_QTILE], h_vis[t]);
     ann[t] = h_n_path ? h_n_path[t] : 0;
     for (int j = 0; j < 4; ++j) an[t * 4 + j] = (h_path_rows && j < ann[t]) ? h_path_rows[t * 4 + j] : 0;
   }
@@ -177,10 +179,11 @@ atspeed_status atspeed_op_attention(atspeed_stream stream, const void* d_q, cons
   a.kv_rows = cache_rows;
   a.n_qtiles = nqt;
   const int off_qt0 = 0, off_qtn = nqt, off_qtu = 2 * nqt, off_tu = 3 * nqt, off_tv = off_tu + T, off_an = off_tv + T,
-            off_ann = off_an + 4 * T, off_pg = off_ann + T, off_sp = off_pg + pages;
+            off_ann = off_an + 4 * T, off_pg = off_ann + T, off_sp = off_pg + pages, off_qtv = off_sp + 1;
   a.qt_t0 = ip + off_qt0;
   a.qt_n = ip + off_qtn;
   a.qt_user = ip + off_qtu;
+  a.qt_vis = ip + off_qtv;
   a.tok_user = ip + off_tu;
   a.tok_vis = ip + off_tv;
   a.anc_row = ip + off_an;
