@@ -65,7 +65,10 @@ struct FLayout {
 
 struct GP {
   int epi;
-  bool to_dh;    // O / down projection: the product goes to dh (the next norm phase adds it to h)
+  bool dh_out;   // O / down projection: the product goes to dh (the next norm phase adds it to h)
+  bool to_dh;    // ... with its split tiles' parts left in the workspace for the norm phase to sum
+                 // (few rows, BN = 128); with BN = 256 (many rows per CTA in the norm) the GEMM
+                 // phase sums them itself
   int M, K, m_tiles, n_tiles, kb, up_row0, rows;  // rows: valid tokens of the phase
   WorkSplit w;   // whole tiles per CTA + stream-K over the remaining tiles
   int mapA, mapB, layer;
@@ -78,6 +81,7 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
   g.layer = gi / 4;
   g.up_row0 = 0;
   g.rows = p.T;
+  g.dh_out = false;
   g.to_dh = false;
   if (gi == 4 * L) {
     g.epi = EPI_F32;
@@ -96,7 +100,8 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
       g.mapB = act0;
     } else if (k == 1) {
       g.epi = EPI_F32;
-      g.to_dh = true;
+      g.dh_out = true;
+      g.to_dh = BN == 128;
       g.M = p.d;
       g.K = p.d;
       g.mapB = act0 + 1;
@@ -108,7 +113,8 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
       g.mapB = act0;
     } else {
       g.epi = EPI_F32;
-      g.to_dh = true;
+      g.dh_out = true;
+      g.to_dh = BN == 128;
       g.M = p.d;
       g.K = p.ffn;
       g.mapB = act0 + 2;
@@ -253,7 +259,7 @@ __device__ GemmArgs epi_args(const FwdParams& p, const GP& g) {
   a.q_out = p.q;
   a.k_cache = p.kc + p.layer_elems * g.layer;
   a.v_cache = p.vc + p.layer_elems * g.layer;
-  if (g.to_dh) {
+  if (g.dh_out) {
     a.out_f32 = p.dh;
     a.ldo = p.d;
   } else if (g.epi == EPI_F32) {
@@ -279,7 +285,7 @@ __device__ void build_part_table(const FwdParams& p, int gi, int nt, int* toff, 
   long long tu0 = 0;
   if (ctid < g.m_tiles) {
     const int t = ctid * g.n_tiles + nt;
-    if (t < g.w.r) {   // a stream-K tile; whole tiles have a single part, written to dh
+    if (t < g.w.r && g.to_dh) {   // a stream-K tile; whole (or GEMM-summed) tiles are in dh
       tu0 = (long long)t * g.kb;
       c_first = sk_owner(g.w, tu0);
       cnt = sk_owner(g.w, tu0 + g.kb - 1) - c_first + 1;
@@ -530,7 +536,8 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       part_slot[pi] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
     }
   };
-  const bool shared_sums = !g.to_dh && (g.w.q > 0 || (gi == 4 * p.L && g.w.Gsk > 0 && g.w.Usk / g.w.Gsk + 1 < kb));
+  const bool shared_sums =
+      !g.to_dh && (g.w.q > 0 || g.dh_out || (gi == 4 * p.L && g.w.Gsk > 0 && g.w.Usk / g.w.Gsk + 1 < kb));
   if (shared_sums && it.u < it.u1) {
     int sk_tile[2], nsk = 0;
     while (it.u < it.u1 && nsk < 2) {
