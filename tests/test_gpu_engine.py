@@ -419,3 +419,38 @@ def test_full_norm_sd_lossless_and_matches_oracle_tiny(ats):
         assert len(set(got)) == w.K and all(g in valid for g in got)
         assert np.all(np.diff(rx_sc[u].cpu().numpy()) <= 0)
     ctx.close()
+
+
+def test_api_errors_are_status_codes(ats):
+    """Wrong calls return status codes (no trap, the context stays usable): options outside the
+    limits, steps before a prefill, a normalisation change inside a step, injected logits under FULL
+    normalisation, FULL-only accessors outside it."""
+    w = synth.workload("tiny")
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    prompt = synth.make_prompts(1, w.prompt_len, w.target.vocab, w.seed)[0]
+    ctx = _ctx(ats, w.target, w.draft, items, w.code_base, 1, len(prompt), w.K, w.N, w.gamma, seed=w.seed)
+    o = ats.opts(w.K, w.N, w.gamma)
+    with pytest.raises(ats.AtSpeedError) as e:
+        ctx.begin_step(o)
+    assert e.value.status == -6                      # E_STATE: no prefill yet
+    _prefill(ats, ctx, [prompt])
+    with pytest.raises(ats.AtSpeedError) as e:
+        ctx.begin_step(ats.opts(w.K + 1, w.N, w.gamma))
+    assert e.value.status == -2                      # E_SHAPE: K above the limit
+    ctx.begin_step(o)
+    with pytest.raises(ats.AtSpeedError) as e:
+        ctx.draft_step(ats.opts(w.K, w.N, w.gamma, norm=ats.NORM_FULL), ats.STRICT)
+    assert e.value.status == -6                      # E_STATE: normalisation changed inside the step
+    with pytest.raises(ats.AtSpeedError) as e:
+        ctx.node_lse(0, 0, 0)
+    assert e.value.status == -1                      # E_ARG: not a FULL step
+    ctx.draft_step(o, ats.STRICT)                    # the context is still usable
+    ctx.close()
+    ctx = _ctx(ats, w.target, w.draft, items, w.code_base, 1, len(prompt), w.K, w.N, w.gamma, seed=w.seed)
+    _prefill(ats, ctx, [prompt])
+    of = ats.opts(w.K, w.N, w.gamma, norm=ats.NORM_FULL)
+    ctx.begin_step(of)
+    with pytest.raises(ats.AtSpeedError) as e:
+        ctx.draft_step_logits(of, ats.STRICT, np.zeros((1, w.K, 1024), np.float32))
+    assert e.value.status == -6                      # E_STATE: injected logits have no whole-vocabulary rows
+    ctx.close()
