@@ -7,8 +7,10 @@
 // takes equal contiguous ranges of units, so every SM streams the same number of weight bytes
 // whatever the matrix shape.  A tile whose k-range spans several CTAs is reduced through an fp32
 // workspace by the last CTA to finish it (fixed summation order, hence deterministic), which then
-// runs the fused epilogue.  The partition depends only on (M, K, tokens rounded to the tile and
-// the grid), so a token's output does not depend on which other tokens share the call.
+// runs the fused epilogue.  The partition depends only on (M, K, the number of token tiles and the
+// grid), so a token's output does not depend on the other tokens of the call as long as the calls
+// compared have the same number of token tiles (one tile up to 256 tokens); with more token tiles
+// the k-split, and so the order of the fp32 sums, can differ.
 //
 // Roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM allocator + MMA issuer, warps 2-5 =
 // epilogue (TMEM lane quadrant = warp % 4).  Two TMEM accumulators alternate between segments so
