@@ -29,7 +29,31 @@ namespace {
 
 thread_local std::string g_create_error;
 
-constexpr int kChunksPerSplit = 2;  // prefix pages per attention split (tree queries)
+// Prefix pages per attention split of a model's tree forwards, fixed per context (so a node's
+// output does not depend on the call it is in): among 1, 2, 4, ... pages, the one that minimises
+// the estimated time of the attention phase -- rounds of work items over the 2 x grid warpgroup
+// slots, each item costing a fixed start (Q, first K / V copy, partials; ~9 us) plus ~2.2 us per
+// page -- for the limits' typical call: max_users users of min(3 max_N, node slots) tree tokens,
+// in query tiles of 64, times the heads.  One user at the bench shape gets 2 pages (256 items in
+// one round); 16 users get whole-prefix items (many rounds, so fewer and longer items win).
+int attention_pages_per_split(const atspeed_limits& L, int H, int grid) {
+  const int pages = std::max(1, (L.max_prompt + ATT_PAGE - 1) / ATT_PAGE);
+  const int stride = L.max_K + L.max_gamma * L.max_N;
+  const int tokens = std::max(1, std::min(3 * L.max_N, stride));
+  const long long pairs = (long long)L.max_users * ((tokens + ATT_QTILE - 1) / ATT_QTILE) * H;
+  int best = 1;
+  double best_t = 1e30;
+  for (int cps = 1; cps < 2 * pages; cps *= 2) {
+    const long long items = pairs * ((pages + cps - 1) / cps);
+    const long long rounds = (items + 2LL * grid - 1) / (2LL * grid);
+    const double t = (double)rounds * (9.0 + 2.2 * std::min(cps, pages));
+    if (t < best_t - 1e-9) {
+      best_t = t;
+      best = cps;
+    }
+  }
+  return best;
+}
 
 struct Fail {
   atspeed_status st;
@@ -39,6 +63,7 @@ struct ModelRt {
   bool present = false;
   bool per_op = false;   // this model's forward runs one kernel per op (else one persistent launch)
   int grid = 0;          // CTAs of its GEMM work splits (both schedules, so both give the same bits)
+  int cps = 2;           // prefix pages per attention split of its tree forwards (fixed per context)
   int layers = 0, d = 0, H = 0, hd = 0, ffn = 0, V = 0;
   float eps = 1e-6f, theta = 1e4f;
   const bf16 *embed = nullptr, *final_norm = nullptr, *lm_head = nullptr;
@@ -323,7 +348,12 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.rows_sel = dalloc<int>(c, m.Tcap);
   m.user_splits = dalloc<int>(c, L.max_users);
   const int pages = c->prefix_pages_per_user;
-  m.max_splits = std::max(1, (pages + kChunksPerSplit - 1) / kChunksPerSplit);
+  {
+    // the grid the model's forward will run on (as set with the schedule) and its split size
+    const int grid = std::max(1, std::min(gemm_grid_size(c->device), 2 * m.ffn / 128));
+    m.cps = attention_pages_per_split(L, m.H, grid);
+  }
+  m.max_splits = std::max(1, (pages + m.cps - 1) / m.cps);
   const int Ttree = std::max(L.max_users * stride, m.Tcap);
   m.part_o = dalloc<float>(c, (size_t)m.max_splits * Ttree * m.d, false);
   m.part_ml = dalloc<float>(c, (size_t)m.max_splits * Ttree * m.H * 2, false);
@@ -596,7 +626,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     a.page_table = c->page_table;
     a.max_pages = c->prefix_pages_per_user;
     a.user_splits = m.user_splits;
-    a.chunks_per_split = p.prefill ? 0 : kChunksPerSplit;
+    a.chunks_per_split = p.prefill ? 0 : m.cps;
     a.max_splits = max_split;
     a.out = m.att;
     a.part_o = m.part_o;
@@ -664,7 +694,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     a.page_table = c->page_table;
     a.max_pages = c->prefix_pages_per_user;
     a.user_splits = m.user_splits;
-    a.chunks_per_split = p.prefill ? 0 : kChunksPerSplit;
+    a.chunks_per_split = p.prefill ? 0 : m.cps;
     a.max_splits = max_split;
     a.out = m.att;
     a.part_o = m.part_o;
@@ -765,9 +795,9 @@ void add_qtiles(FwdPlan& p, int u, int t0, int n, int vis) {
   }
 }
 
-int splits_for(int P) {
+int splits_for(int P, int cps) {
   const int pages = (P + ATT_PAGE - 1) / ATT_PAGE;
-  return std::max(1, (pages + kChunksPerSplit - 1) / kChunksPerSplit);
+  return std::max(1, (pages + cps - 1) / cps);
 }
 
 // Forward of the given node slots of the current step through model m (target or draft).
@@ -794,7 +824,7 @@ void forward_nodes(atspeed_ctx* c, ModelRt& m, bool target, const std::vector<in
     i = j;
   }
   p.splits.resize(c->B);
-  for (int u = 0; u < c->B; ++u) p.splits[u] = splits_for(c->users[u].P);
+  for (int u = 0; u < c->B; ++u) p.splits[u] = splits_for(c->users[u].P, m.cps);
   p.out_rows.resize(T);
   for (int k = 0; k < T; ++k) p.out_rows[k] = k;
   p.logit_row_base = row_base;
