@@ -69,6 +69,9 @@ def parse():
     ap.add_argument("--norm", choices=["masked", "full"], default="masked",
                     help="constrained log-softmax normaliser: the valid children (default) or the whole "
                          "vocabulary (the LM head then runs over all V rows)")
+    ap.add_argument("--early-reject", action="store_true",
+                    help="decide level 1 of depth-0 steps from the prefill logits and skip the tree forward "
+                         "when every user rejects it (same outputs; not part of the paper's method)")
     ap.add_argument("--verify-only", type=int, default=0, metavar="R",
                     help="profiling aid: R verification calls of the workload, each in an NVTX range 'verify'")
     ap.add_argument("--layers", type=int, default=0, metavar="L",
@@ -260,6 +263,7 @@ def run_ours(args, w):
         if world > 1:
             dist.barrier()
 
+    ctx.set_early_reject(args.early_reject)
     # ---- warm-up, then K timed steps (inputs resident in HBM)
     for _ in range(args.warmup):
         ctx.beam_search(toks, offsets, o, mode)
@@ -297,7 +301,9 @@ def run_ours(args, w):
     e2e = {"value": job_rate(B, world, args.steps, ms_e2e), "unit": "rec lists/s",
            "h2d_bytes_per_step": int(h_tok.numel() * 4), "d2h_bytes_per_step": int(h_items.numel() * 4 + h_sc.numel() * 4)}
 
-    # ---- the verification call alone (first call of a decode: depth 0, T = 3 N tree tokens)
+    # ---- the verification call alone (first call of a decode: depth 0, T = 3 N tree tokens); always
+    # the full call, whatever --early-reject says
+    ctx.set_early_reject(False)
     hbm, tf, tf_sus, peak_kind = peaks()
     ver_ms, fk = [], {"ms": 0.0, "launches": 0}
     n_timed = max(3, args.steps)
@@ -342,7 +348,8 @@ def run_ours(args, w):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights, synthetic items)",
         "config": {"workload": f"{w.name}: 7B-shape target (32L d4096 H32 ffn11008 V33024), draft 4L d768, "
                                f"K={w.K} N={w.N} gamma={w.gamma}, P={w.prompt_len[0]}, {w.n_items} Zipf items, "
-                               f"{args.mode} verification, {args.norm} normalisation, {B} user(s) per GPU",
+                               f"{args.mode} verification, {args.norm} normalisation, {B} user(s) per GPU"
+                               + (", early rejection at depth 0" if args.early_reject else ""),
                    "l2": "inputs larger than L2 (13.5 GB of target weights per verification call)"},
         "roofline": dict(roof, **{
             "traffic": TRAFFIC_PER_ALG_BYTE * vb,
@@ -356,6 +363,7 @@ def run_ours(args, w):
         "verify_call": {"ms": v_ms, "tree_tokens": T_first, "alg_bytes": vb, "alg_flops": vf,
                         "t_roof_ms": t_roof, "frac_of_roofline": t_roof / v_ms, "peak_source": peak_kind},
         "accepted_steps_per_list": float(np.mean(stats[:, 0])), "verify_calls_per_list": float(np.mean(stats[:, 1])),
+        "tree_tokens_per_list": float(np.mean(stats[:, 2])),
         "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
     }
     if rank == 0 and world == 1:

@@ -163,6 +163,17 @@ atspeed_status atspeed_beam_search(atspeed_ctx *ctx, atspeed_stream stream, int 
                                    const int32_t *h_offsets, const atspeed_decode_opts *opts,
                                    atspeed_decode_mode mode, int32_t *d_items, float *d_scores, int32_t *h_stats);
 
+/* Early rejection (off by default; not part of the paper's method, same outputs bit for bit).
+ * At depth 0 the target logits of the empty beam come from the prefill, so the acceptance of
+ * drafted level 1 (Alg. 1: are the top-K of level 1 all drafted?  Alg. 2: is |A| >= K?) can be
+ * decided before any forward over the tree.  When every active user rejects level 1 -- its output
+ * beams are then level-1 candidates scored from those logits alone -- the step ends without the
+ * target forward (and, in atspeed_beam_search, without drafting levels 2 .. gamma).  Such a step
+ * counts as a verification call with 0 tree tokens.  Costs one extra verification launch and one
+ * host synchronisation per depth-0 step when some user accepts.  ATSPEED_E_STATE while a step is
+ * open. */
+atspeed_status atspeed_set_early_reject(atspeed_ctx *ctx, int enable);
+
 /* ----------------------------------------------------------------------------------------------
  * Introspection / test hooks.
  * ---------------------------------------------------------------------------------------------- */

@@ -24,7 +24,7 @@ PLAIN_TOPK, PLAIN_SAMPLE, SD_STRICT, SD_RELAXED = 0, 1, 2, 3
 EXPORTS = [
     "atspeed_create", "atspeed_destroy", "atspeed_last_error", "atspeed_prefill", "atspeed_begin_step",
     "atspeed_draft_step", "atspeed_verify", "atspeed_draft_step_logits", "atspeed_verify_logits",
-    "atspeed_beam_search", "atspeed_profile", "atspeed_profile_read", "atspeed_tree_shape", "atspeed_debug_tree",
+    "atspeed_beam_search", "atspeed_set_early_reject", "atspeed_profile", "atspeed_profile_read", "atspeed_tree_shape", "atspeed_debug_tree",
     "atspeed_debug_node_logits", "atspeed_debug_node_lse", "atspeed_debug_buffer", "atspeed_set_tree", "atspeed_op_workspace_bytes", "atspeed_op_gemm",
     "atspeed_op_gemm_noalloc", "atspeed_op_gemm_swiglu", "atspeed_op_rmsnorm", "atspeed_op_attention_scratch", "atspeed_op_attention",
 ]
@@ -86,6 +86,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "atspeed_draft_step_logits": (c_int, [vp, vp, ctypes.POINTER(DecodeOpts), c_int, fp]),
         "atspeed_verify_logits": (c_int, [vp, vp, ctypes.POINTER(DecodeOpts), c_int, fp, vp, vp, vp, vp]),
         "atspeed_beam_search": (c_int, [vp, vp, c_int, vp, i32p, ctypes.POINTER(DecodeOpts), c_int, vp, vp, i32p]),
+        "atspeed_set_early_reject": (c_int, [vp, c_int]),
         "atspeed_profile": (c_int, [vp, c_int]),
         "atspeed_profile_read": (c_int, [vp, c_int, i32p, ctypes.POINTER(ctypes.c_double),
                                          ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]),
@@ -249,6 +250,9 @@ class Context:
                                              mode, items.data_ptr(), scores.data_ptr(),
                                              stats.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))), self.ptr)
         return items, scores, stats
+
+    def set_early_reject(self, enable: bool):
+        _check(self._lib.atspeed_set_early_reject(self.ptr, 1 if enable else 0), self.ptr)
 
     def profile(self, enable: bool):
         _check(self._lib.atspeed_profile(self.ptr, 1 if enable else 0), self.ptr)

@@ -156,6 +156,8 @@ struct atspeed_ctx {
   bool full_norm = false;      // the current step normalises over the whole vocabulary (FULL)
   int step_K = 0, step_N = 0, step_gamma = 0, levels_done = 0;
   bool roots_drafted = false;
+  bool level_fwd_pending = false;  // the draft forward of level `levels_done` has not run yet
+  bool early_reject = false;       // decide level 1 of depth-0 steps before any forward over it
   bool tree_injected = false;
   bool have_tree = false;      // a node table exists (debug hooks may read it)
   std::vector<UserState> users;
@@ -920,6 +922,7 @@ void open_step(atspeed_ctx* c, const atspeed_decode_opts* o, cudaStream_t st) {
   c->have_tree = true;
   c->levels_done = 0;
   c->roots_drafted = false;
+  c->level_fwd_pending = false;
   c->tree_injected = false;
 }
 
@@ -975,7 +978,20 @@ std::vector<int> level_nodes(atspeed_ctx* c, int lvl, bool need_forward_rule) {
   return v;
 }
 
-void draft_step_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts* o, atspeed_verify_mode mode) {
+// Draft forward over the nodes of drafted level `lvl` (their logits draft level lvl + 1).
+void draft_level_forward(atspeed_ctx* c, int lvl, cudaStream_t st) {
+  std::vector<int> nodes = level_nodes(c, lvl, true);
+  // rows of this level's draft logits follow the rows already used in this step
+  int base = c->B + (int)level_nodes(c, 0, false).size();
+  for (int j = 1; j < lvl; ++j) base += (int)level_nodes(c, j, true).size();
+  forward_nodes(c, c->drf, false, nodes, base, st);
+  c->level_fwd_pending = false;
+}
+
+// forward_level = false leaves the draft forward over the new level pending: the next draft_step
+// or verify runs it, an early-rejected step never does.
+void draft_step_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts* o, atspeed_verify_mode mode,
+                     bool forward_level = true) {
   check_opts(c, o);
   if (!c->drf.present) {
     set_err(c, "no draft model in this context");
@@ -986,7 +1002,7 @@ void draft_step_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts*
     set_err(c, "the tree of this step was injected");
     throw Fail{ATSPEED_E_STATE};
   }
-  const int stride = c->step_K + c->step_gamma * c->step_N;
+  if (c->level_fwd_pending) draft_level_forward(c, c->levels_done, st);
   // draft logits rows: users' prefill rows first, then one row per node slot
   if (!c->roots_drafted) {
     std::vector<int> roots = level_nodes(c, 0, false);
@@ -1001,13 +1017,11 @@ void draft_step_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts*
   const TreeDev t = tree_dev(c);
   CK(draft_level_launch(t, lvl, c->step_N, mode == ATSPEED_RELAXED, o->philox_seed, st, c->pdl));
   c->n_launch += 1;
-  std::vector<int> nodes = level_nodes(c, lvl, true);
-  // rows of this level's draft logits follow the rows already used in this step
-  int base = c->B + (int)level_nodes(c, 0, false).size();
-  for (int j = 1; j < lvl; ++j) base += (int)level_nodes(c, j, true).size();
-  forward_nodes(c, c->drf, false, nodes, base, st);
   c->levels_done = lvl;
-  (void)stride;
+  if (forward_level)
+    draft_level_forward(c, lvl, st);
+  else
+    c->level_fwd_pending = true;
 }
 
 void commit(atspeed_ctx* c, cudaStream_t st, bool count_stats, const std::vector<int>& T_user) {
@@ -1059,9 +1073,48 @@ void commit(atspeed_ctx* c, cudaStream_t st, bool count_stats, const std::vector
   c->step_open = false;
 }
 
-void verify_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts* o, atspeed_verify_mode mode) {
+// Early rejection (opt-in, atspeed_set_early_reject).  At depth 0 the target logits of level 0 (the
+// empty beam) are the prefill's, so whether drafted level 1 is accepted can be decided before any
+// forward over the tree.  A user that rejects level 1 takes its K output beams from level 1's
+// candidates (Alg. 1: the top-K of level 1; Alg. 2: A plus draws from the residual), which depend
+// on those logits alone: when every active user rejects, the tree forward is skipped and the step
+// ends with the same outputs as the full verification.
+bool early_reject_eligible(const atspeed_ctx* c) {
+  if (!c->early_reject || c->levels_done < 1) return false;
+  bool any = false;
+  for (const auto& us : c->users) {
+    if (!us.active) continue;
+    if (us.d != 0 || us.g < 1) return false;
+    any = true;
+  }
+  return any;
+}
+
+// One probe launch of the verification kernel; true when every active user was decided at level 1
+// (its outputs are then in the o_* buffers, ready for commit).
+bool early_reject_probe(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts* o, atspeed_verify_mode mode) {
+  const TreeDev t = tree_dev(c);
+  VerifyOut vo{c->o_acc, c->o_adv, c->o_n, c->o_nacc, c->o_path, c->o_score, c->o_parent, c->o_trie};
+  CK(verify_launch(t, c->step_K, mode == ATSPEED_RELAXED, o->philox_seed, vo, st, c->pdl, true));
+  c->n_launch += 1;
+  std::vector<int> acc(c->B);
+  CK(cudaMemcpyAsync(acc.data(), c->o_acc, c->B * 4, cudaMemcpyDeviceToHost, st));
+  CK(cudaStreamSynchronize(st));
+  for (int u = 0; u < c->B; ++u)
+    if (c->users[u].active && acc[u] < 0) return false;
+  return true;
+}
+
+void verify_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts* o, atspeed_verify_mode mode,
+                 bool allow_probe = true) {
   check_opts(c, o);
   ensure_step(c, o, st);
+  if (allow_probe && early_reject_eligible(c) && early_reject_probe(c, st, o, mode)) {
+    c->level_fwd_pending = false;
+    commit(c, st, true, std::vector<int>(c->B, 0));
+    return;
+  }
+  if (c->level_fwd_pending) draft_level_forward(c, c->levels_done, st);
   // target forward over the incoming beams (depth >= 1) and drafted levels 1 .. min(g, L-d-1)
   std::vector<int> nodes;
   std::vector<int> T_user(c->B, 0);
@@ -1470,10 +1523,22 @@ atspeed_status atspeed_beam_search(atspeed_ctx* c, atspeed_stream stream, int n_
       int maxg = 0;
       for (auto& us : c->users)
         if (us.active) maxg = std::max(maxg, us.g);
-      for (int j = 0; j < maxg; ++j) draft_step_impl(c, st, &o, vm);
+      // with early rejection the level-1 decision is taken right after drafting level 1, before the
+      // draft forward over it: a step that every user rejects at level 1 runs no further forward
+      const bool probe = c->early_reject && maxg >= 1;
+      bool decided = false;
       std::vector<bool> was(n_users);
       for (int u = 0; u < n_users; ++u) was[u] = c->users[u].active;
-      verify_impl(c, st, &o, vm);
+      for (int j = 0; j < maxg && !decided; ++j) {
+        draft_step_impl(c, st, &o, vm, !(probe && j == 0));
+        if (probe && j == 0 && early_reject_eligible(c) && early_reject_probe(c, st, &o, vm)) decided = true;
+      }
+      if (decided) {
+        c->level_fwd_pending = false;
+        commit(c, st, true, std::vector<int>(n_users, 0));
+      } else {
+        verify_impl(c, st, &o, vm, !probe);
+      }
       for (int u = 0; u < n_users; ++u)
         if (was[u] && !c->users[u].active) {
           fin_path[u] = c->users[u].path;
@@ -1508,6 +1573,16 @@ atspeed_status atspeed_begin_step(atspeed_ctx* c, atspeed_stream stream, const a
       throw Fail{ATSPEED_E_STATE};
     }
     ensure_step(c, opts, (cudaStream_t)stream);
+  });
+}
+
+atspeed_status atspeed_set_early_reject(atspeed_ctx* c, int enable) {
+  return guarded(c, [&] {
+    if (c->step_open) {
+      set_err(c, "set_early_reject: a speculative step is open");
+      throw Fail{ATSPEED_E_STATE};
+    }
+    c->early_reject = enable != 0;
   });
 }
 

@@ -20,8 +20,10 @@ cudaError_t rmsnorm_rows_launch(const float* h, const int* rows, int n, const __
 size_t select_smem_bytes(int max_parents);
 cudaError_t draft_level_launch(const TreeDev& t, int lvl, int N, bool relaxed, uint64_t seed, cudaStream_t st,
                                bool pdl);
+// probe: decide level 1 only (see verify_strict_kernel); users whose level 1 is accepted get
+// accepted = -1 and must be verified again by a full launch
 cudaError_t verify_launch(const TreeDev& t, int K, bool relaxed, uint64_t seed, const VerifyOut& o, cudaStream_t st,
-                          bool pdl);
+                          bool pdl, bool probe = false);
 
 // Per-token inputs of a forward over tree nodes, read from the node table.
 struct FwdTokens {

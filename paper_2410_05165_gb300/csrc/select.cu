@@ -351,9 +351,12 @@ __global__ void __launch_bounds__(NT) draft_level_kernel(TreeDev t, int lvl, int
 }
 
 // ---------------------------------------------------------------------------------------------
-// strict top-K verification (Alg. 1); g = 0 gives one step of plain target beam search
+// strict top-K verification (Alg. 1); g = 0 gives one step of plain target beam search.
+// probe != 0 (g >= 1): only level 1 is examined -- a user whose level 1 is rejected gets its
+// complete output exactly as in the full call (it depends on the level-0 logits alone); a user
+// whose level 1 is accepted gets accepted = -1 and nothing else.
 // ---------------------------------------------------------------------------------------------
-__global__ void __launch_bounds__(NT) verify_strict_kernel(TreeDev t, int K, VerifyOut o) {
+__global__ void __launch_bounds__(NT) verify_strict_kernel(TreeDev t, int K, VerifyOut o, int probe) {
   extern __shared__ uint8_t sm[];
   __shared__ Scratch s;
   __shared__ int sel[256], tmp[256];
@@ -421,6 +424,10 @@ __global__ void __launch_bounds__(NT) verify_strict_kernel(TreeDev t, int K, Ver
       if (f < 0) atomicAnd(&all_ok, 0);
     }
     __syncthreads();
+    if (probe && all_ok) {
+      if (threadIdx.x == 0) o.accepted[u] = -1;
+      return;
+    }
     if (!all_ok) {
       a = j - 1;
       adv = j;
@@ -466,9 +473,12 @@ __global__ void __launch_bounds__(NT) verify_strict_kernel(TreeDev t, int K, Ver
 }
 
 // ---------------------------------------------------------------------------------------------
-// relaxed sampling verification (Sec. 3.2, Alg. 2); g = 0 gives one step of sampling beam search
+// relaxed sampling verification (Sec. 3.2, Alg. 2); g = 0 gives one step of sampling beam search.
+// probe != 0 (g >= 1): as in the strict kernel, a user whose level 1 is rejected (|A| < K) gets
+// its complete output, one whose level 1 is accepted gets accepted = -1.
 // ---------------------------------------------------------------------------------------------
-__global__ void __launch_bounds__(NT) verify_relaxed_kernel(TreeDev t, int K, VerifyOut o, uint64_t seed) {
+__global__ void __launch_bounds__(NT) verify_relaxed_kernel(TreeDev t, int K, VerifyOut o, uint64_t seed,
+                                                            int probe) {
   extern __shared__ uint8_t sm[];
   __shared__ Scratch s;
   __shared__ int sel[256], tmp[256];
@@ -561,6 +571,10 @@ __global__ void __launch_bounds__(NT) verify_relaxed_kernel(TreeDev t, int K, Ve
     if (f) accd[pos] = threadIdx.x;
     __syncthreads();
     nacc_last = na;
+    if (probe && na >= K) {
+      if (threadIdx.x == 0) o.accepted[u] = -1;
+      return;
+    }
     if (na >= K) {
       if (j < g) {
         // step accepted: the drafted beams of level j carry their target scores to step j + 1
@@ -705,18 +719,18 @@ cudaError_t draft_level_launch(const TreeDev& t, int lvl, int N, bool relaxed, u
 }
 
 cudaError_t verify_launch(const TreeDev& t, int K, bool relaxed, uint64_t seed, const VerifyOut& o, cudaStream_t st,
-                          bool pdl) {
+                          bool pdl, bool probe) {
   const size_t smem = select_smem_bytes(max(t.slots_in, t.slots_lvl));
   cudaLaunchAttribute at[1];
   cudaLaunchConfig_t c = cfg_for(t.B, smem, st, at, pdl);
   if (relaxed) {
     cudaError_t e = set_smem(verify_relaxed_kernel, smem);
     if (e != cudaSuccess) return e;
-    return cudaLaunchKernelEx(&c, verify_relaxed_kernel, t, K, o, seed);
+    return cudaLaunchKernelEx(&c, verify_relaxed_kernel, t, K, o, seed, probe ? 1 : 0);
   }
   cudaError_t e = set_smem(verify_strict_kernel, smem);
   if (e != cudaSuccess) return e;
-  return cudaLaunchKernelEx(&c, verify_strict_kernel, t, K, o);
+  return cudaLaunchKernelEx(&c, verify_strict_kernel, t, K, o, probe ? 1 : 0);
 }
 
 }  // namespace atspeed

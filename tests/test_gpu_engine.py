@@ -421,6 +421,59 @@ def test_full_norm_sd_lossless_and_matches_oracle_tiny(ats):
     ctx.close()
 
 
+@pytest.mark.parametrize("mode", ["SD_STRICT", "SD_RELAXED"])
+@pytest.mark.parametrize("self_draft", [False, True])
+def test_early_reject_same_outputs(ats, mode, self_draft):
+    """Early rejection changes no output bit: beam_search and the explicit draft/verify calls return
+    the same beams, scores, accepted lengths and call counts with it on and off.  With an unrelated
+    draft level 1 is rejected at depth 0 and tree tokens drop; with the target as its own draft
+    level 1 is accepted, the probe hands over to the full verification and nothing is skipped."""
+    w = synth.workload("tiny")
+    B = 3
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    prompts = synth.make_prompts(B, w.prompt_len, w.target.vocab, w.seed)
+    tw = ats.weights_to_device(synth.model_weights(w.target, w.seed, "target"))
+    if self_draft:
+        d_spec, dw = w.target, tw
+    else:
+        d_spec, dw = w.draft, ats.weights_to_device(synth.model_weights(w.draft, w.seed, "draft"))
+    ctx = ats.Context(w.target, tw, d_spec, dw, items, w.code_base, max_users=B, max_prompt=32, max_K=w.K,
+                      max_N=w.N, max_gamma=w.gamma)
+    toks = torch.from_numpy(np.concatenate(prompts)).cuda()
+    off = np.concatenate([[0], np.cumsum([len(p) for p in prompts])]).astype(np.int32)
+    m = getattr(ats, mode)
+    vm = ats.STRICT if mode == "SD_STRICT" else ats.RELAXED
+    o = ats.opts(w.K, w.N, w.gamma, seed=11)
+    ref_items, ref_sc, ref_st = ctx.beam_search(toks, off, o, m)
+    ctx.set_early_reject(True)
+    got_items, got_sc, got_st = ctx.beam_search(toks, off, o, m)
+    np.testing.assert_array_equal(got_items.cpu().numpy(), ref_items.cpu().numpy())
+    np.testing.assert_array_equal(got_sc.cpu().numpy(), ref_sc.cpu().numpy())
+    np.testing.assert_array_equal(got_st[:, :2], ref_st[:, :2])
+    assert np.all(got_st[:, 2] <= ref_st[:, 2])
+    if self_draft and mode == "SD_STRICT":
+        np.testing.assert_array_equal(got_st, ref_st)   # level 1 always accepted: nothing skipped
+    elif not self_draft:
+        assert got_st[:, 2].sum() < ref_st[:, 2].sum()
+    # explicit calls: one depth-0 step (every level drafted and forwarded, only the target forward
+    # can be skipped), the same outputs on and off
+    outs = []
+    for er in (False, True):
+        ctx.set_early_reject(er)
+        ctx.prefill(toks, off)
+        for _ in range(w.gamma):
+            ctx.draft_step(o, vm)
+        outs.append([x.cpu().numpy() for x in ctx.verify(o, vm)])
+    for a, b in zip(*outs):
+        np.testing.assert_array_equal(a, b)
+    with pytest.raises(ats.AtSpeedError) as e:
+        ctx.prefill(toks, off)
+        ctx.begin_step(o)
+        ctx.set_early_reject(False)
+    assert e.value.status == -6                      # E_STATE: not inside a step
+    ctx.close()
+
+
 def test_api_errors_are_status_codes(ats):
     """Wrong calls return status codes (no trap, the context stays usable): options outside the
     limits, steps before a prefill, a normalisation change inside a step, injected logits under FULL
