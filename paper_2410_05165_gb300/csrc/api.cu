@@ -101,6 +101,7 @@ struct ModelRt {
   const bf16** d_attn_norm = nullptr;    // device arrays of layer pointers
   const bf16** d_mlp_norm = nullptr;
   int* att_counters = nullptr;
+  int* plan_blk = nullptr;   // qt_* / user_splits / rows_sel of the current forward, packed
   int max_qt = 0;
 };
 
@@ -145,6 +146,17 @@ struct atspeed_ctx {
   float *n_sq = nullptr, *n_sp = nullptr;
   int *u_d = nullptr, *u_g = nullptr, *u_step = nullptr, *u_P = nullptr, *page_table = nullptr;
   int* fwd_nodes = nullptr;
+  // pinned host staging for uploads and downloads: regions are handed out in order and reclaimed
+  // at the next synchronisation of the stream (every copy staged before it has then completed)
+  uint8_t* h_stage = nullptr;
+  size_t stage_cap = 0, stage_used = 0;
+  int* n_blk = nullptr;     // node table: the n_* arrays, packed for the current step's size
+  int* u_blk = nullptr;     // per-user d, g, step, P (max_users each)
+  int* o_blk = nullptr;     // verification outputs (fixed sections, max_users x max_K)
+  int* o_anc_t = nullptr;   // [max_users][max_K][4] ancestor rows of the output beams' parents
+  int* o_anc_d = nullptr;
+  int* fwd_zero = nullptr;  // grid barrier, split arrivals and attention arrivals, zeroed per forward
+  size_t fwd_zero_att = 0;  // offset of the attention arrivals in fwd_zero
   // verify outputs
   int *o_acc = nullptr, *o_adv = nullptr, *o_n = nullptr, *o_nacc = nullptr, *o_path = nullptr, *o_parent = nullptr,
       *o_trie = nullptr;
@@ -225,16 +237,72 @@ T* dalloc(atspeed_ctx* c, size_t n, bool zero = true) {
   return static_cast<T*>(p);
 }
 
+void stage_sync(atspeed_ctx* c, cudaStream_t st);
+template <typename T>
+T* stage_alloc(atspeed_ctx* c, cudaStream_t st, size_t n);
+
+// Synchronises the stream and reads the device error word (one download through the staging
+// buffer; regions staged before the call stay readable until the next staging request).
 void check_device_error(atspeed_ctx* c, cudaStream_t st) {
-  CK(cudaStreamSynchronize(st));
-  unsigned int w = 0;
-  CK(cudaMemcpy(&w, c->err_word, sizeof w, cudaMemcpyDeviceToHost));
+  unsigned int* hw = stage_alloc<unsigned int>(c, st, 1);
+  CK(cudaMemcpyAsync(hw, c->err_word, sizeof(unsigned int), cudaMemcpyDeviceToHost, st));
+  stage_sync(c, st);
+  const unsigned int w = *hw;
   if (w) {
     CK(cudaMemset(c->err_word, 0, sizeof w));
     set_err(c, "device error word 0x%x (%s)", w, (w & ATSPEED_DEV_ERR_TIMEOUT) ? "bounded wait timed out" : "bounds");
     throw Fail{(w & ATSPEED_DEV_ERR_TIMEOUT) ? ATSPEED_E_TIMEOUT : ATSPEED_E_CUDA};
   }
 }
+
+void stage_sync(atspeed_ctx* c, cudaStream_t st) {
+  CK(cudaStreamSynchronize(st));
+  c->stage_used = 0;
+}
+
+// A region of the pinned staging buffer that stays untouched until the stream's next
+// synchronisation by stage_sync (which the next region may force when the buffer is full).
+template <typename T>
+T* stage_alloc(atspeed_ctx* c, cudaStream_t st, size_t n) {
+  const size_t bytes = (n * sizeof(T) + 255) & ~size_t(255);
+  if (bytes > c->stage_cap) {
+    set_err(c, "staging request of %zu bytes exceeds the %zu-byte staging buffer", bytes, c->stage_cap);
+    throw Fail{ATSPEED_E_SHAPE};
+  }
+  if (c->stage_used + bytes > c->stage_cap) stage_sync(c, st);
+  T* p = reinterpret_cast<T*>(c->h_stage + c->stage_used);
+  c->stage_used += bytes;
+  return p;
+}
+
+// Host-to-device copy through the staging buffer (the source may be freed on return).
+void upload(atspeed_ctx* c, cudaStream_t st, void* dst, const void* src, size_t bytes) {
+  if (bytes == 0) return;
+  uint8_t* h = stage_alloc<uint8_t>(c, st, bytes);
+  memcpy(h, src, bytes);
+  CK(cudaMemcpyAsync(dst, h, bytes, cudaMemcpyHostToDevice, st));
+}
+
+// Points the n_* arrays at consecutive sections of the node-table block for n slots and B users
+// of g drafted levels (one contiguous upload in open_step).
+void carve_nodes(atspeed_ctx* c, size_t n, int B, int g) {
+  int* q = c->n_blk;
+  c->n_code = q, q += n;
+  c->n_prank = q, q += n;
+  c->n_trie = q, q += n;
+  c->n_path = q, q += 4 * n;
+  c->n_row_t = q, q += n;
+  c->n_row_d = q, q += n;
+  c->n_anc_t = q, q += 4 * n;
+  c->n_anc_d = q, q += 4 * n;
+  c->n_lg_t = q, q += n;
+  c->n_lg_d = q, q += n;
+  c->n_sq = reinterpret_cast<float*>(q), q += n;
+  c->n_sp = reinterpret_cast<float*>(q), q += n;
+  c->n_cnt = q, q += (size_t)B * (g + 1);
+}
+constexpr size_t NODE_INTS = 21;   // ints per slot in the node table (the n_* arrays above)
+size_t o_blk_ints(int mu, int mK) { return 4 * (size_t)mu + 15 * (size_t)mu * mK; }
 
 void init_model(atspeed_ctx* c, ModelRt& m, const atspeed_model_desc* md, const char* name) {
   if (!md) return;
@@ -343,12 +411,7 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.ancn = dalloc<int>(c, m.Tcap);
   const int max_qt = m.Tcap / ATT_QTILE + L.max_users + 1;
   char eb[256];
-  m.qt_t0 = dalloc<int>(c, max_qt);
-  m.qt_n = dalloc<int>(c, max_qt);
-  m.qt_user = dalloc<int>(c, max_qt);
-  m.qt_vis = dalloc<int>(c, max_qt);
-  m.rows_sel = dalloc<int>(c, m.Tcap);
-  m.user_splits = dalloc<int>(c, L.max_users);
+  m.plan_blk = dalloc<int>(c, 4 * (size_t)max_qt + L.max_users + m.Tcap);   // carved per forward
   const int pages = c->prefix_pages_per_user;
   {
     // the grid the model's forward will run on (as set with the schedule) and its split size
@@ -359,8 +422,7 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   const int Ttree = std::max(L.max_users * stride, m.Tcap);
   m.part_o = dalloc<float>(c, (size_t)m.max_splits * Ttree * m.d, false);
   m.part_ml = dalloc<float>(c, (size_t)m.max_splits * Ttree * m.H * 2, false);
-  m.max_qt = max_qt;
-  m.att_counters = dalloc<int>(c, (size_t)max_qt * m.H);
+  m.max_qt = max_qt;   // (the attention arrival counters live in the ctx's per-forward zero block)
   // tensor maps of the persistent forward
   const int nmaps = fwd_map_count(m.layers);
   std::vector<CUtensorMap> hm(nmaps);
@@ -563,12 +625,28 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     throw Fail{ATSPEED_E_SHAPE};
   }
   const int nqt = (int)p.qt_t0.size();
-  CK(cudaMemcpyAsync(m.qt_t0, p.qt_t0.data(), nqt * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(m.qt_n, p.qt_n.data(), nqt * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(m.qt_user, p.qt_user.data(), nqt * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(m.qt_vis, p.qt_vis.data(), nqt * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(m.user_splits, p.splits.data(), p.splits.size() * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(m.rows_sel, p.out_rows.data(), p.out_rows.size() * 4, cudaMemcpyHostToDevice, st));
+  if (nqt > m.max_qt || (int)p.splits.size() > c->lim.max_users || (int)p.out_rows.size() > m.Tcap) {
+    set_err(c, "forward plan exceeds capacity (%d query tiles, %zu users, %zu rows)", nqt, p.splits.size(),
+            p.out_rows.size());
+    throw Fail{ATSPEED_E_SHAPE};
+  }
+  {
+    // the plan's tables, packed: one upload into the model's plan block
+    const size_t ns = p.splits.size(), nr = p.out_rows.size(), tot = 4 * (size_t)nqt + ns + nr;
+    int* h = stage_alloc<int>(c, st, tot);
+    int* q = h;
+    for (const std::vector<int>* v : {&p.qt_t0, &p.qt_n, &p.qt_user, &p.qt_vis, &p.splits, &p.out_rows}) {
+      memcpy(q, v->data(), v->size() * sizeof(int));
+      q += v->size();
+    }
+    m.qt_t0 = m.plan_blk;
+    m.qt_n = m.qt_t0 + nqt;
+    m.qt_user = m.qt_n + nqt;
+    m.qt_vis = m.qt_user + nqt;
+    m.user_splits = m.qt_vis + nqt;
+    m.rows_sel = m.user_splits + ns;
+    CK(cudaMemcpyAsync(m.plan_blk, h, tot * sizeof(int), cudaMemcpyHostToDevice, st));
+  }
   int max_split = 1;
   for (int s : p.splits) max_split = std::max(max_split, s);
   const size_t per = (size_t)m.rows * m.d;
@@ -643,9 +721,7 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     f.bar = c->fwd_bar;
     f.err = c->err_word;
     f.trace = c->fwd_trace;
-    CK(cudaMemsetAsync(c->fwd_bar, 0, sizeof(unsigned int), st));
-    CK(cudaMemsetAsync(m.att_counters, 0, (size_t)nqt * m.H * sizeof(int), st));
-    CK(cudaMemsetAsync(c->fwd_sk, 0, (size_t)(4 * m.layers + 1) * c->fwd_grid * sizeof(int), st));
+    CK(cudaMemsetAsync(c->fwd_zero, 0, (c->fwd_zero_att + (size_t)nqt * m.H) * sizeof(int), st));
     if (c->fwd_trace) CK(cudaMemsetAsync(c->fwd_trace, 0, c->fwd_trace_n * sizeof(unsigned long long), st));
     const double wbytes = 2.0 * m.layers * (4.0 * m.d * m.d + 3.0 * m.d * m.ffn) + 2.0 * ITEM_ROWS * m.d;
     ProfScope ps(c, st, 6, wbytes, 2.0 * T * (wbytes / 2.0));
@@ -808,7 +884,7 @@ void forward_nodes(atspeed_ctx* c, ModelRt& m, bool target, const std::vector<in
   if (nodes.empty()) return;
   const int T = (int)nodes.size();
   const TreeDev t = tree_dev(c);
-  CK(cudaMemcpyAsync(c->fwd_nodes, nodes.data(), T * 4, cudaMemcpyHostToDevice, st));
+  upload(c, st, c->fwd_nodes, nodes.data(), (size_t)T * 4);
   FwdTokens f{m.tok, m.pos, m.kvrow, m.tuser, m.tvis, m.anc, m.ancn};
   CK(tree_gather_launch(t, c->fwd_nodes, T, c->u_P, c->code_base, target, row_base, f, st, c->pdl));
   c->n_launch += 1;
@@ -838,19 +914,16 @@ void forward_nodes(atspeed_ctx* c, ModelRt& m, bool target, const std::vector<in
 // speculative-step bookkeeping
 // ---------------------------------------------------------------------------------------------
 void upload_users(atspeed_ctx* c, cudaStream_t st) {
-  std::vector<int> d(c->B), g(c->B), s(c->B), P(c->B);
+  const int mu = c->lim.max_users;
+  int* h = stage_alloc<int>(c, st, 4 * (size_t)mu);
   for (int u = 0; u < c->B; ++u) {
     const UserState& us = c->users[u];
-    d[u] = us.active ? us.d : TREE_L;
-    g[u] = us.active ? us.g : 0;
-    s[u] = us.step;
-    P[u] = us.P;
+    h[u] = us.active ? us.d : TREE_L;
+    h[mu + u] = us.active ? us.g : 0;
+    h[2 * mu + u] = us.step;
+    h[3 * mu + u] = us.P;
   }
-  CK(cudaMemcpyAsync(c->u_d, d.data(), c->B * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->u_g, g.data(), c->B * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->u_step, s.data(), c->B * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->u_P, P.data(), c->B * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaStreamSynchronize(st));  // host vectors are stack-local
+  CK(cudaMemcpyAsync(c->u_blk, h, 4 * (size_t)mu * sizeof(int), cudaMemcpyHostToDevice, st));
 }
 
 // Writes level 0 (incoming beams) and the own-row assignment of every slot of the new step.
@@ -861,9 +934,31 @@ void open_step(atspeed_ctx* c, const atspeed_decode_opts* o, cudaStream_t st) {
   c->step_gamma = G;
   const int stride = K + G * N;
   const size_t n = (size_t)c->B * stride;
-  std::vector<int> code(n, -1), prank(n, -1), trie(n, 0), path(n * 4, -1), rt(n), rd(n), at(n * 4, 0), ad(n * 4, 0),
-      lgt(n, -1), lgd(n, -1), cnt((size_t)c->B * (G + 1), 0);
-  std::vector<float> sq(n, -INFINITY), sp(n, -INFINITY);
+  // the node table of this step: n slots in consecutive sections, filled in the staging buffer and
+  // uploaded at once
+  const size_t ncnt = (size_t)c->B * (G + 1);
+  carve_nodes(c, n, c->B, G);
+  int* h = stage_alloc<int>(c, st, NODE_INTS * n + ncnt);
+  int* code = h;
+  int* prank = code + n;
+  int* trie = prank + n;
+  int* path = trie + n;
+  int* rt = path + 4 * n;
+  int* rd = rt + n;
+  int* at = rd + n;
+  int* ad = at + 4 * n;
+  int* lgt = ad + 4 * n;
+  int* lgd = lgt + n;
+  float* sq = reinterpret_cast<float*>(lgd + n);
+  float* sp = sq + n;
+  int* cnt = reinterpret_cast<int*>(sp + n);
+  std::fill(code, code + 3 * n, -1);           // code, prank: -1
+  std::fill(trie, trie + n, 0);
+  std::fill(path, path + 4 * n, -1);
+  std::fill(at, at + 8 * n, 0);                // at, ad
+  std::fill(lgt, lgt + 2 * n, -1);             // lg_t, lg_d
+  std::fill(sq, sq + 2 * n, -INFINITY);        // sq, sp
+  std::fill(cnt, cnt + ncnt, 0);
   for (int u = 0; u < c->B; ++u) {
     UserState& us = c->users[u];
     us.g = us.active ? std::min(G, TREE_L - us.d) : 0;
@@ -895,19 +990,7 @@ void open_step(atspeed_ctx* c, const atspeed_decode_opts* o, cudaStream_t st) {
       }
     }
   }
-  CK(cudaMemcpyAsync(c->n_code, code.data(), n * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_prank, prank.data(), n * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_trie, trie.data(), n * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_path, path.data(), n * 16, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_row_t, rt.data(), n * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_row_d, rd.data(), n * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_anc_t, at.data(), n * 16, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_anc_d, ad.data(), n * 16, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_lg_t, lgt.data(), n * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_lg_d, lgd.data(), n * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_sq, sq.data(), n * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_sp, sp.data(), n * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->n_cnt, cnt.data(), cnt.size() * 4, cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->n_blk, h, (NODE_INTS * n + ncnt) * sizeof(int), cudaMemcpyHostToDevice, st));
   c->full_norm = o->norm == ATSPEED_NORM_FULL;
   if (c->full_norm) {
     // level 0 of users at depth 0 scores with the prefill's logits rows 0 .. B-1
@@ -917,7 +1000,7 @@ void open_step(atspeed_ctx* c, const atspeed_decode_opts* o, cudaStream_t st) {
       for (ModelRt* m : {&c->tgt, &c->drf})
         if (m->present) full_lse(c, *m, m->root_x, m->root_rows, c->B, m->lse, st);
   }
-  upload_users(c, st);  // synchronises (host vectors above are local)
+  upload_users(c, st);
   c->step_open = true;
   c->have_tree = true;
   c->levels_done = 0;
@@ -1026,20 +1109,22 @@ void draft_step_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts*
 
 void commit(atspeed_ctx* c, cudaStream_t st, bool count_stats, const std::vector<int>& T_user) {
   const int B = c->B, K = c->step_K;
-  const int stride = c->step_K + c->step_gamma * c->step_N;
-  std::vector<int> acc(B), adv(B), nout(B), path((size_t)B * K * 4), parent((size_t)B * K), trie((size_t)B * K);
-  std::vector<float> score((size_t)B * K);
-  std::vector<int> anc_t((size_t)B * stride * 4), anc_d((size_t)B * stride * 4);
-  CK(cudaMemcpyAsync(acc.data(), c->o_acc, B * 4, cudaMemcpyDeviceToHost, st));
-  CK(cudaMemcpyAsync(adv.data(), c->o_adv, B * 4, cudaMemcpyDeviceToHost, st));
-  CK(cudaMemcpyAsync(nout.data(), c->o_n, B * 4, cudaMemcpyDeviceToHost, st));
-  CK(cudaMemcpyAsync(path.data(), c->o_path, path.size() * 4, cudaMemcpyDeviceToHost, st));
-  CK(cudaMemcpyAsync(parent.data(), c->o_parent, parent.size() * 4, cudaMemcpyDeviceToHost, st));
-  CK(cudaMemcpyAsync(trie.data(), c->o_trie, trie.size() * 4, cudaMemcpyDeviceToHost, st));
-  CK(cudaMemcpyAsync(score.data(), c->o_score, score.size() * 4, cudaMemcpyDeviceToHost, st));
-  CK(cudaMemcpyAsync(anc_t.data(), c->n_anc_t, anc_t.size() * 4, cudaMemcpyDeviceToHost, st));
-  CK(cudaMemcpyAsync(anc_d.data(), c->n_anc_d, anc_d.size() * 4, cudaMemcpyDeviceToHost, st));
-  check_device_error(c, st);
+  // every output section in one download (fixed section offsets: max_users, max_K)
+  const int mu = c->lim.max_users;
+  const size_t mk = (size_t)mu * c->lim.max_K, nblk = o_blk_ints(mu, c->lim.max_K);
+  int* h = stage_alloc<int>(c, st, nblk);
+  CK(cudaMemcpyAsync(h, c->o_blk, nblk * sizeof(int), cudaMemcpyDeviceToHost, st));
+  check_device_error(c, st);   // synchronises; the download stays intact until the next staging
+  const int* adv = h + mu;
+  const int* acc = h;
+  const int* nout = h + 2 * mu;
+  const int* path = h + 4 * mu;
+  const int* parent = path + 4 * mk;
+  const int* trie = parent + mk;
+  const float* score = reinterpret_cast<const float*>(trie + mk);
+  const int* anc_t = reinterpret_cast<const int*>(score + mk);
+  const int* anc_d = anc_t + 4 * mk;
+  (void)parent;
   for (int u = 0; u < B; ++u) {
     UserState& us = c->users[u];
     if (!us.active) continue;
@@ -1054,10 +1139,9 @@ void commit(atspeed_ctx* c, cudaStream_t st, bool count_stats, const std::vector
       for (int i = 0; i < 4; ++i) us.path[k][i] = path[o * 4 + i];
       us.sp[k] = score[o];
       us.trie[k] = trie[o];
-      const int par = parent[o];
       for (int i = 0; i < 4; ++i) {
-        us.anc_t[k][i] = i < nd - 1 ? anc_t[(size_t)par * 4 + i] : 0;
-        us.anc_d[k][i] = i < nd - 1 ? anc_d[(size_t)par * 4 + i] : 0;
+        us.anc_t[k][i] = i < nd - 1 ? anc_t[o * 4 + i] : 0;
+        us.anc_d[k][i] = i < nd - 1 ? anc_d[o * 4 + i] : 0;
       }
     }
     if (count_stats) {
@@ -1094,12 +1178,13 @@ bool early_reject_eligible(const atspeed_ctx* c) {
 // (its outputs are then in the o_* buffers, ready for commit).
 bool early_reject_probe(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts* o, atspeed_verify_mode mode) {
   const TreeDev t = tree_dev(c);
-  VerifyOut vo{c->o_acc, c->o_adv, c->o_n, c->o_nacc, c->o_path, c->o_score, c->o_parent, c->o_trie};
+  VerifyOut vo{c->o_acc, c->o_adv, c->o_n, c->o_nacc, c->o_path, c->o_score, c->o_parent, c->o_trie,
+               c->o_anc_t, c->o_anc_d};
   CK(verify_launch(t, c->step_K, mode == ATSPEED_RELAXED, o->philox_seed, vo, st, c->pdl, true));
   c->n_launch += 1;
-  std::vector<int> acc(c->B);
-  CK(cudaMemcpyAsync(acc.data(), c->o_acc, c->B * 4, cudaMemcpyDeviceToHost, st));
-  CK(cudaStreamSynchronize(st));
+  int* acc = stage_alloc<int>(c, st, c->B);
+  CK(cudaMemcpyAsync(acc, c->o_acc, c->B * 4, cudaMemcpyDeviceToHost, st));
+  stage_sync(c, st);
   for (int u = 0; u < c->B; ++u)
     if (c->users[u].active && acc[u] < 0) return false;
   return true;
@@ -1143,7 +1228,8 @@ void verify_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts* o, 
   for (int n : nodes) T_user[n / stride] += 1;
   forward_nodes(c, c->tgt, true, nodes, c->B, st);
   const TreeDev t = tree_dev(c);
-  VerifyOut vo{c->o_acc, c->o_adv, c->o_n, c->o_nacc, c->o_path, c->o_score, c->o_parent, c->o_trie};
+  VerifyOut vo{c->o_acc, c->o_adv, c->o_n, c->o_nacc, c->o_path, c->o_score, c->o_parent, c->o_trie,
+               c->o_anc_t, c->o_anc_d};
   CK(verify_launch(t, c->step_K, mode == ATSPEED_RELAXED, o->philox_seed, vo, st, c->pdl));
   c->n_launch += 1;
   commit(c, st, true, T_user);
@@ -1196,17 +1282,16 @@ void prefill_impl(atspeed_ctx* c, cudaStream_t st, int n_users, const int32_t* d
   p.logit_row_base = 0;
   for (ModelRt* m : {&c->tgt, &c->drf}) {
     if (!m->present) continue;
-    CK(cudaMemcpyAsync(m->pos, pos.data(), T * 4, cudaMemcpyHostToDevice, st));
-    CK(cudaMemcpyAsync(m->kvrow, kvrow.data(), T * 4, cudaMemcpyHostToDevice, st));
-    CK(cudaMemcpyAsync(m->tuser, tuser.data(), T * 4, cudaMemcpyHostToDevice, st));
-    CK(cudaMemcpyAsync(m->tvis, tvis.data(), T * 4, cudaMemcpyHostToDevice, st));
+    upload(c, st, m->pos, pos.data(), (size_t)T * 4);
+    upload(c, st, m->kvrow, kvrow.data(), (size_t)T * 4);
+    upload(c, st, m->tuser, tuser.data(), (size_t)T * 4);
+    upload(c, st, m->tvis, tvis.data(), (size_t)T * 4);
     forward(c, *m, p, st);
     // the last history tokens' final-norm rows, for a FULL-normalised first step
     CK(cudaMemcpyAsync(m->root_x, m->x, (size_t)n_users * m->d * sizeof(bf16), cudaMemcpyDeviceToDevice, st));
   }
-  std::vector<int> Pu(P);
-  CK(cudaMemcpyAsync(c->u_P, Pu.data(), n_users * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaStreamSynchronize(st));
+  upload(c, st, c->u_P, P.data(), (size_t)n_users * 4);
+  stage_sync(c, st);
   c->prefilled = true;
   c->step_open = false;
 }
@@ -1221,7 +1306,7 @@ void inject_logits(atspeed_ctx* c, bool target, int off, int width, const float*
   int* lg = target ? c->n_lg_t : c->n_lg_d;
   const size_t n = (size_t)c->B * stride;
   std::vector<int> rows(n);
-  CK(cudaStreamSynchronize(st));
+  stage_sync(c, st);
   CK(cudaMemcpy(rows.data(), lg, n * 4, cudaMemcpyDeviceToHost));
   for (int u = 0; u < c->B; ++u) {
     if (!c->users[u].active) continue;
@@ -1257,7 +1342,7 @@ void draft_step_logits_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decod
   CK(draft_level_launch(t, lvl, c->step_N, mode == ATSPEED_RELAXED, o->philox_seed, st, c->pdl));
   c->levels_done = lvl;
   c->roots_drafted = true;
-  CK(cudaStreamSynchronize(st));
+  stage_sync(c, st);
 }
 
 void verify_logits_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_opts* o, atspeed_verify_mode mode,
@@ -1280,7 +1365,8 @@ void verify_logits_impl(atspeed_ctx* c, cudaStream_t st, const atspeed_decode_op
   }
   inject_logits(c, true, 0, stride, h_logits, (size_t)stride * ITEM_ROWS, st);
   const TreeDev t = tree_dev(c);
-  VerifyOut vo{c->o_acc, c->o_adv, c->o_n, c->o_nacc, c->o_path, c->o_score, c->o_parent, c->o_trie};
+  VerifyOut vo{c->o_acc, c->o_adv, c->o_n, c->o_nacc, c->o_path, c->o_score, c->o_parent, c->o_trie,
+               c->o_anc_t, c->o_anc_d};
   CK(verify_launch(t, c->step_K, mode == ATSPEED_RELAXED, o->philox_seed, vo, st, c->pdl));
   commit(c, st, true, std::vector<int>(c->B, 0));
 }
@@ -1310,11 +1396,11 @@ void write_outputs(atspeed_ctx* c, cudaStream_t st, int32_t* d_acc, int32_t* d_d
       sc[(size_t)u * K + k] = us.sp[k];
     }
   }
-  if (d_acc) CK(cudaMemcpyAsync(d_acc, acc.data(), B * 4, cudaMemcpyHostToDevice, st));
-  if (d_depth) CK(cudaMemcpyAsync(d_depth, depth.data(), B * 4, cudaMemcpyHostToDevice, st));
-  if (d_beams) CK(cudaMemcpyAsync(d_beams, beams.data(), beams.size() * 4, cudaMemcpyHostToDevice, st));
-  if (d_scores) CK(cudaMemcpyAsync(d_scores, sc.data(), sc.size() * 4, cudaMemcpyHostToDevice, st));
-  CK(cudaStreamSynchronize(st));
+  if (d_acc) upload(c, st, d_acc, acc.data(), (size_t)B * 4);
+  if (d_depth) upload(c, st, d_depth, depth.data(), (size_t)B * 4);
+  if (d_beams) upload(c, st, d_beams, beams.data(), beams.size() * 4);
+  if (d_scores) upload(c, st, d_scores, sc.data(), sc.size() * 4);
+  stage_sync(c, st);
 }
 
 }  // namespace
@@ -1377,11 +1463,19 @@ atspeed_status atspeed_create(const atspeed_model_desc* target, const atspeed_mo
         mr->grid = std::max(1, std::min(c->fwd_grid, 2 * mr->ffn / 128));
       }
     }
-    c->fwd_bar = dalloc<unsigned int>(c, 1);
     {
+      // grid barrier, split-tile arrivals and attention split arrivals of the persistent forward:
+      // one block, zeroed by one memset before every launch
       const int Lmax = std::max(c->tgt.layers, c->drf.present ? c->drf.layers : 0);
       c->fwd_sk_n = (size_t)(4 * Lmax + 1) * c->fwd_grid;
-      c->fwd_sk = dalloc<int>(c, c->fwd_sk_n);
+      size_t att = 0;
+      for (ModelRt* mr : {&c->tgt, &c->drf})
+        if (mr->present) att = std::max(att, (size_t)mr->max_qt * mr->H);
+      c->fwd_zero_att = 32 + c->fwd_sk_n;
+      c->fwd_zero = dalloc<int>(c, c->fwd_zero_att + att);
+      c->fwd_bar = reinterpret_cast<unsigned int*>(c->fwd_zero);
+      c->fwd_sk = c->fwd_zero + 32;
+      for (ModelRt* mr : {&c->tgt, &c->drf}) mr->att_counters = c->fwd_zero + c->fwd_zero_att;
     }
     {
       const char* tr = getenv("ATSPEED_FWD_TRACE");
@@ -1399,36 +1493,43 @@ atspeed_status atspeed_create(const atspeed_model_desc* target, const atspeed_mo
     c->gs.err = c->err_word;
     const size_t nn = (size_t)lim->max_users * stride;
     c->cap_nodes = (int)nn;
-    c->n_code = dalloc<int>(c, nn);
-    c->n_prank = dalloc<int>(c, nn);
-    c->n_trie = dalloc<int>(c, nn);
-    c->n_path = dalloc<int>(c, nn * 4);
-    c->n_row_t = dalloc<int>(c, nn);
-    c->n_row_d = dalloc<int>(c, nn);
-    c->n_anc_t = dalloc<int>(c, nn * 4);
-    c->n_anc_d = dalloc<int>(c, nn * 4);
-    c->n_lg_t = dalloc<int>(c, nn);
-    c->n_lg_d = dalloc<int>(c, nn);
-    c->n_sq = dalloc<float>(c, nn);
-    c->n_sp = dalloc<float>(c, nn);
-    c->n_cnt = dalloc<int>(c, (size_t)lim->max_users * (lim->max_gamma + 1));
-    c->u_d = dalloc<int>(c, lim->max_users);
-    c->u_g = dalloc<int>(c, lim->max_users);
-    c->u_step = dalloc<int>(c, lim->max_users);
-    c->u_P = dalloc<int>(c, lim->max_users);
+    const size_t n_cnt_max = (size_t)lim->max_users * (lim->max_gamma + 1);
+    c->n_blk = dalloc<int>(c, NODE_INTS * nn + n_cnt_max);
+    carve_nodes(c, nn, lim->max_users, lim->max_gamma);
+    const int mu = lim->max_users;
+    c->u_blk = dalloc<int>(c, 4 * (size_t)mu);
+    c->u_d = c->u_blk;
+    c->u_g = c->u_blk + mu;
+    c->u_step = c->u_blk + 2 * mu;
+    c->u_P = c->u_blk + 3 * mu;
     c->fwd_nodes = dalloc<int>(c, nn);
+    // staging: the largest per-step upload is the node table; forward plans and outputs are small
+    c->stage_cap = 2 * (NODE_INTS * nn + n_cnt_max) * sizeof(int) + ((size_t)1 << 20);
+    {
+      void* hp = nullptr;
+      CK(cudaMallocHost(&hp, c->stage_cap));
+      c->h_stage = static_cast<uint8_t*>(hp);
+    }
     std::vector<int> pt((size_t)lim->max_users * c->prefix_pages_per_user);
     for (size_t i = 0; i < pt.size(); ++i) pt[i] = (int)i;  // user u's prefix pages are contiguous
     c->page_table = dalloc<int>(c, pt.size(), false);
     CK(cudaMemcpy(c->page_table, pt.data(), pt.size() * 4, cudaMemcpyHostToDevice));
-    c->o_acc = dalloc<int>(c, lim->max_users);
-    c->o_adv = dalloc<int>(c, lim->max_users);
-    c->o_n = dalloc<int>(c, lim->max_users);
-    c->o_nacc = dalloc<int>(c, lim->max_users);
-    c->o_path = dalloc<int>(c, (size_t)lim->max_users * lim->max_K * 4);
-    c->o_parent = dalloc<int>(c, (size_t)lim->max_users * lim->max_K);
-    c->o_trie = dalloc<int>(c, (size_t)lim->max_users * lim->max_K);
-    c->o_score = dalloc<float>(c, (size_t)lim->max_users * lim->max_K);
+    {
+      // verification outputs in one block, read back by one copy per step
+      const size_t mk = (size_t)mu * lim->max_K;
+      c->o_blk = dalloc<int>(c, o_blk_ints(mu, lim->max_K));
+      int* q = c->o_blk;
+      c->o_acc = q, q += mu;
+      c->o_adv = q, q += mu;
+      c->o_n = q, q += mu;
+      c->o_nacc = q, q += mu;
+      c->o_path = q, q += 4 * mk;
+      c->o_parent = q, q += mk;
+      c->o_trie = q, q += mk;
+      c->o_score = reinterpret_cast<float*>(q), q += mk;
+      c->o_anc_t = q, q += 4 * mk;
+      c->o_anc_d = q, q += 4 * mk;
+    }
     CK(cudaDeviceSynchronize());
   } catch (const Fail& e) {
     g_create_error = c->err;
@@ -1449,6 +1550,7 @@ void atspeed_destroy(atspeed_ctx* c) {
   }
   for (auto e : c->prof_pool) cudaEventDestroy(e);
   for (void* p : c->allocs) cudaFree(p);
+  if (c->h_stage) cudaFreeHost(c->h_stage);
   delete c;
 }
 
@@ -1553,15 +1655,15 @@ atspeed_status atspeed_beam_search(atspeed_ctx* c, atspeed_stream stream, int n_
         for (int i = 0; i < 4; ++i) items[((size_t)u * K + k) * 4 + i] = fin_path[u][k][i];
         sc[(size_t)u * K + k] = fin_sp[u][k];
       }
-    if (d_items) CK(cudaMemcpyAsync(d_items, items.data(), items.size() * 4, cudaMemcpyHostToDevice, st));
-    if (d_scores) CK(cudaMemcpyAsync(d_scores, sc.data(), sc.size() * 4, cudaMemcpyHostToDevice, st));
+    if (d_items) upload(c, st, d_items, items.data(), items.size() * 4);
+    if (d_scores) upload(c, st, d_scores, sc.data(), sc.size() * 4);
     if (h_stats)
       for (int u = 0; u < n_users; ++u) {
         h_stats[u * 3 + 0] = c->users[u].acc_steps;
         h_stats[u * 3 + 1] = c->users[u].calls;
         h_stats[u * 3 + 2] = c->users[u].tree_tokens;
       }
-    CK(cudaStreamSynchronize(st));
+    stage_sync(c, st);
   });
 }
 
@@ -1740,7 +1842,7 @@ atspeed_status atspeed_set_tree(atspeed_ctx* c, atspeed_stream stream, int n_lev
     std::vector<int> code(n), prank(n), trie(n), path(n * 4), rt(n), rd(n), at(n * 4), ad(n * 4), lgd(n),
         cnt((size_t)c->B * (G + 1));
     std::vector<float> sq(n), sp(n);
-    CK(cudaStreamSynchronize(st));
+    stage_sync(c, st);
     CK(cudaMemcpy(code.data(), c->n_code, n * 4, cudaMemcpyDeviceToHost));
     CK(cudaMemcpy(trie.data(), c->n_trie, n * 4, cudaMemcpyDeviceToHost));
     CK(cudaMemcpy(path.data(), c->n_path, n * 16, cudaMemcpyDeviceToHost));

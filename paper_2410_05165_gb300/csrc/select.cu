@@ -279,6 +279,10 @@ __device__ void write_out(const TreeDev& t, const VerifyOut& o, int K, int u, in
   o.out_score[(size_t)u * K + r] = score;
   o.out_parent[(size_t)u * K + r] = parent;
   o.out_trie[(size_t)u * K + r] = trie_child(t, t.trie[parent], c);
+  for (int i = 0; i < TREE_L; ++i) {
+    o.out_anc_t[((size_t)u * K + r) * 4 + i] = t.anc_t[(size_t)parent * 4 + i];
+    o.out_anc_d[((size_t)u * K + r) * 4 + i] = t.anc_d[(size_t)parent * 4 + i];
+  }
 }
 
 // ---------------------------------------------------------------------------------------------

@@ -59,6 +59,8 @@ struct VerifyOut {
   float* out_score;    // [B][K]
   int* out_parent;     // [B][K] global node index of the output beam's parent
   int* out_trie;       // [B][K] trie node of the output beam's prefix
+  int* out_anc_t;      // [B][K][4] target cache rows of the parent's path tokens (anc_t of the parent)
+  int* out_anc_d;      // [B][K][4] the same in the draft cache
 };
 
 }  // namespace atspeed

@@ -128,6 +128,41 @@ def test_decode_logic_bit_exact_on_synthetic_logits(ats, K, N, G, mode):
     ctx.close()
 
 
+def _sparse_items(kind):
+    """Degenerate catalogues: fewer items than beams, or one shared first code (level 1 has a
+    single candidate, later levels a handful)."""
+    if kind == "fewer_than_K":
+        return synth.make_items(7, "uniform", 1.1, 5)
+    rng = np.random.default_rng(21)
+    rest = rng.choice(256 ** 3, size=15, replace=False)
+    return np.stack([np.full(15, 5), rest // 65536, rest // 256 % 256, rest % 256], axis=1).astype(np.int32)
+
+
+@pytest.mark.parametrize("kind", ["fewer_than_K", "shared_prefix"])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_decode_logic_sparse_trie(ats, kind, mode):
+    """Levels with fewer valid extensions than K or N: drafting keeps only the valid children, the
+    output holds every item when there are fewer than K (missing beams padded), and the decode
+    equals oracle.sd_decode bit for bit (items, accepted lengths) with scores within 1e-4."""
+    items = _sparse_items(kind)
+    trie = Trie(items)
+    spec = synth.ModelSpec(1, 64, 2, 128, 1024)
+    B, K, N, G, philox = 2, 10, 20, 3, 777
+    ctx = _ctx(ats, spec, spec, items, 0, B, 16, K, N, G)
+    _prefill(ats, ctx, [np.arange(4 + u, dtype=np.int32) for u in range(B)])
+    fin, steps = _drive_logits_decode(ats, ctx, B, K, N, G, mode, 300, 400, philox)
+    for u in range(B):
+        ref, ref_sc, st = sd_decode(rows_fn(300, u), rows_fn(400, u), trie, K, N, G,
+                                    "relaxed" if mode == 1 else "strict", seed=philox, user=u)
+        got, got_sc = fin[u]
+        assert got == ref, (u, got, ref)
+        assert len(got) == min(K, len(items))
+        np.testing.assert_allclose(got_sc[:len(ref)], ref_sc, rtol=0, atol=1e-4)
+        assert np.all(np.isneginf(got_sc[len(ref):]))
+        assert [a for (_, a) in steps[u]] == [s[1] for s in st.steps]
+    ctx.close()
+
+
 @pytest.mark.parametrize("sample", [False, True])
 def test_plain_beam_search_logic_on_synthetic_logits(ats, sample):
     """gamma = 0: plain top-K beam search (strict) / sampling beam search (relaxed)."""
