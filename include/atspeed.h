@@ -19,9 +19,11 @@
  *     borrowed and must stay alive and unchanged until atspeed_destroy.
  *   - Work is enqueued on the given stream (a cudaStream_t; NULL is the legacy default stream).
  *     Calls that must read results back (verify, beam_search) synchronise that stream.
- *   - One context is not thread-safe; use one context per stream.  Every GPU buffer the context
- *     needs (KV caches, node pool, activations, workspace) is allocated once in atspeed_create,
- *     sized by atspeed_limits.
+ *   - One context is not thread-safe; use one context per stream, and pass that same stream to
+ *     every call on it (host-to-device copies go through a pinned staging buffer of the context
+ *     that is reused after the stream's next synchronisation).  Every GPU buffer the context
+ *     needs (KV caches, node pool, activations, workspace) and the staging buffer are allocated
+ *     once in atspeed_create, sized by atspeed_limits.
  *   - Token id of code c at identifier level l (0-based) is code_base + 256 * l + c.
  */
 #ifndef ATSPEED_H_
