@@ -361,7 +361,7 @@ def _near_tie_level(item_rows, full_rows, trie, K, tol):
     from oracle.beam import child_paths, expand, topk
     beams, sp = [()], np.zeros(1, np.float32)
     for _ in range(L):
-        C = expand(beams, sp, item_rows(beams), trie, full_rows(beams))
+        C = expand(beams, sp, item_rows(beams), trie, full_rows(beams) if full_rows else None)
         sc = np.sort(C.score.astype(np.float64))[::-1]
         if sc.size > K and sc[K - 1] - sc[K] < tol:
             return True
@@ -507,6 +507,57 @@ def test_early_reject_same_outputs(ats, mode, self_draft):
         ctx.set_early_reject(False)
     assert e.value.status == -6                      # E_STATE: not inside a step
     ctx.close()
+
+
+def test_mid_full_size_lists_match_oracle(ats):
+    """The mid workload at full size (16 layers, d 2048, V 33 024, 256-token history, 20 000 Zipf
+    items, K = 10, N = 40, gamma = 4, strict): speculative decoding equals the plain target beam
+    search bit for bit on the GPU, and the list is the oracle's plain beam search up to near-ties.
+
+    Tolerance: the node-logit checks bound the GPU's bf16 forward at 2e-2 mean absolute logit error;
+    a beam score adds L = 4 masked log-probs, each off by its code's logit error minus the shift of
+    the children's log-sum-exp, so an item's score is held to L x 2.5e-2 = 0.1 of the oracle's.  Two
+    items may swap ranks only when their oracle scores are within twice that, and the set may differ
+    only when some level's K-th and (K+1)-th oracle candidates are within it."""
+    import scipy.special
+    w = synth.workload("mid")
+    items = synth.make_items(w.n_items, w.code_dist, w.zipf_a, w.seed)
+    prompt = synth.make_prompts(1, w.prompt_len, w.target.vocab, w.seed)[0]
+    tw_np = synth.model_weights(w.target, w.seed, "target")
+    ctx = ats.Context(w.target, ats.weights_to_device(tw_np), w.draft,
+                      ats.weights_to_device(synth.model_weights(w.draft, w.seed, "draft")), items, w.code_base,
+                      max_users=1, max_prompt=len(prompt), max_K=w.K, max_N=w.N, max_gamma=w.gamma)
+    toks = torch.from_numpy(prompt.astype(np.int32)).cuda()
+    o = ats.opts(w.K, w.N, w.gamma)
+    sd_items, sd_sc, stats = ctx.beam_search(toks, [0, len(prompt)], o, ats.SD_STRICT)
+    pl_items, pl_sc, _ = ctx.beam_search(toks, [0, len(prompt)], o, ats.PLAIN_TOPK)
+    ctx.close()
+    np.testing.assert_array_equal(sd_items.cpu().numpy(), pl_items.cpu().numpy())
+    np.testing.assert_array_equal(sd_sc.cpu().numpy(), pl_sc.cpu().numpy())
+    assert stats[0, 1] >= 1
+    trie = Trie(items)
+    ev = PathEvaluator(Model(w.target, tw_np, w.code_base), prompt)
+    item_rows = lambda ps: [r[256 * len(p):256 * (len(p) + 1)].astype(np.float32) for p, r in zip(ps, ev.logits(ps))]
+    ref, ref_sc = plain_beam_search(item_rows, trie, w.K)
+    got = [tuple(int(c) for c in r) for r in sd_items[0].cpu().numpy()]
+    got_sc = sd_sc[0].cpu().numpy()
+    tol = L * 2.5e-2
+
+    def oracle_score(it):
+        s = 0.0
+        for l in range(L):
+            r = item_rows([it[:l]])[0].astype(np.float64)
+            s += r[it[l]] - scipy.special.logsumexp(r[trie.children(it[:l])])
+        return s
+    osc = [oracle_score(it) for it in got]
+    for it, g, r in zip(got, got_sc, osc):
+        assert abs(float(g) - r) < tol, (it, g, r)
+    if set(got) == set(ref):
+        for i in range(len(got)):
+            for j in range(i + 1, len(got)):
+                assert osc[i] > osc[j] - 2 * tol, (got[i], got[j], osc[i], osc[j])
+    else:
+        assert _near_tie_level(item_rows, None, trie, w.K, tol), (got, ref)
 
 
 def test_api_errors_are_status_codes(ats):
