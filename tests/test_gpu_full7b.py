@@ -9,7 +9,8 @@ one layer):
   search, bit for bit (same logits, same ranking);
 * the persistent forward and the one-kernel-per-op forward give the same tree-node logits, bit for
   bit, on the verification call;
-* relaxed speculative decoding returns K distinct valid items ranked by target score.
+* relaxed speculative decoding returns K distinct valid items ranked by target score, also for the
+  16-user workload (ragged 256-1 024-token histories, K = 20, N = 80), reproducibly per seed.
 """
 import numpy as np
 import pytest
@@ -122,3 +123,33 @@ def test_7b_sweep_points_strict_lossless(ats, world, B, K, gamma, N, full):
     np.testing.assert_array_equal(sd_sc.cpu().numpy(), pl_sc.cpu().numpy())
     assert sd_items.shape == (B, K, 4)
     ctx.close()
+
+
+def test_7b_b16_relaxed_config_valid_and_reproducible(ats, world):
+    """The 16-user workload the bench's second line times (histories of 256 to 1 024 tokens, 200 000
+    Zipf items, K = 20, N = 80, gamma = 4, relaxed verification with per-user Philox streams):
+    every user gets K distinct valid items ranked by target score, and a second decode with the same
+    seed reproduces every list bit for bit; with another seed some list changes."""
+    w7 = synth.workload("7b_b16")
+    items = synth.make_items(w7.n_items, w7.code_dist, w7.zipf_a, w7.seed)
+    prompts = synth.make_prompts(w7.n_users, w7.prompt_len, w7.target.vocab, w7.seed)
+    P = [len(p) for p in prompts]
+    assert min(P) >= 256 and max(P) <= 1024 and len(set(P)) > 1   # ragged histories
+    ctx = ats.Context(w7.target, world[1], w7.draft, world[2], items, w7.code_base, max_users=w7.n_users,
+                      max_prompt=max(P), max_K=w7.K, max_N=w7.N, max_gamma=w7.gamma)
+    toks = torch.from_numpy(np.concatenate(prompts).astype(np.int32)).cuda()
+    off = np.concatenate([[0], np.cumsum(P)]).astype(np.int32).tolist()
+    o = ats.opts(w7.K, w7.N, w7.gamma, w7.philox_seed)
+    a_items, a_sc, stats = ctx.beam_search(toks, off, o, ats.SD_RELAXED)
+    b_items, b_sc, _ = ctx.beam_search(toks, off, o, ats.SD_RELAXED)
+    c_items, _, _ = ctx.beam_search(toks, off, ats.opts(w7.K, w7.N, w7.gamma, w7.philox_seed + 1), ats.SD_RELAXED)
+    ctx.close()
+    np.testing.assert_array_equal(a_items.cpu().numpy(), b_items.cpu().numpy())
+    np.testing.assert_array_equal(a_sc.cpu().numpy(), b_sc.cpu().numpy())
+    assert not np.array_equal(a_items.cpu().numpy(), c_items.cpu().numpy())
+    valid = {tuple(int(c) for c in it) for it in items}
+    for u in range(w7.n_users):
+        got = [tuple(int(c) for c in r) for r in a_items[u].cpu().numpy()]
+        assert len(set(got)) == w7.K and all(g in valid for g in got), u
+        assert np.all(np.diff(a_sc[u].cpu().numpy()) <= 0), u
+    assert np.all(stats[:, 1] >= 1)
