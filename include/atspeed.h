@@ -262,7 +262,7 @@ atspeed_status atspeed_op_gemm_noalloc(atspeed_stream stream, const void *d_W, c
                                        int x_rows, float *d_Y, int ldy, int accumulate);
 
 /* out[t][j] = bf16(silu(G[t][j]) * U[t][j]) with G = X W[0:F]^T, U = X W[F:2F]^T (SwiGLU), W bf16
- * [2F][K]; out bf16 [T][ldo]. */
+ * [2F][K]; out bf16 [T][ldo] with ldo even and d_out 4-byte aligned (ATSPEED_E_ARG otherwise). */
 atspeed_status atspeed_op_gemm_swiglu(atspeed_stream stream, const void *d_W, const void *d_X, int F, int K, int T,
                                       int x_rows, void *d_out, int ldo, void *d_ws);
 

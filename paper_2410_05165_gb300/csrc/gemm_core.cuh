@@ -179,25 +179,30 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, in
       }
     }
   } else if constexpr (EPI == EPI_SWIGLU) {
-    // thread owns feature i of the tile and tokens (ep_tid >> 6) + 2k.  silu(g) = g / (1 + e^-g)
-    // with the hardware exponential and an approximate divide (a few ulp, far below the bf16
-    // rounding of the product; for g -> -inf the divisor overflows to inf and the quotient is -0);
-    // the IEEE expf and divide made this loop latency-bound (about 2 us per 32-token chunk)
-    const int i = ep_tid & 63, n0 = ep_tid >> 6;
-    __nv_bfloat16* out = a.out_bf16 + m_tile * 64 + i;
+    // thread owns features 2f, 2f + 1 of the tile (one 4-byte store per token) and tokens
+    // (ep_tid >> 5) + 4k.  silu(g) = g / (1 + e^-g) with the hardware exponential and an
+    // approximate divide (a few ulp, far below the bf16 rounding of the product; for g -> -inf the
+    // divisor overflows to inf and the quotient is -0); the IEEE expf and divide made this loop
+    // latency-bound (about 2 us per 32-token chunk)
+    const int f = ep_tid & 31, n0 = ep_tid >> 5;
+    __nv_bfloat16* out = a.out_bf16 + m_tile * 64 + 2 * f;
     const int T = a.T;
     const size_t ldo = (size_t)a.ldo;
-    float gv[16], uv[16];
+    float2 gv[8], uv[8];
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      const int n = n0 + 2 * k;
-      gv[k] = st[n * GEMM_BM + i];
-      uv[k] = st[n * GEMM_BM + 64 + i];
+    for (int k = 0; k < 8; ++k) {
+      const int n = n0 + 4 * k;
+      gv[k] = *reinterpret_cast<const float2*>(st + n * GEMM_BM + 2 * f);
+      uv[k] = *reinterpret_cast<const float2*>(st + n * GEMM_BM + 64 + 2 * f);
     }
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      const int tok = tok0 + n0 + 2 * k;
-      if (tok < T) out[(size_t)tok * ldo] = __float2bfloat16_rn(__fdividef(gv[k], 1.0f + __expf(-gv[k])) * uv[k]);
+    for (int k = 0; k < 8; ++k) {
+      const int tok = tok0 + n0 + 4 * k;
+      if (tok < T) {
+        const float y0 = __fdividef(gv[k].x, 1.0f + __expf(-gv[k].x)) * uv[k].x;
+        const float y1 = __fdividef(gv[k].y, 1.0f + __expf(-gv[k].y)) * uv[k].y;
+        *reinterpret_cast<__nv_bfloat162*>(out + (size_t)tok * ldo) = __floats2bfloat162_rn(y0, y1);
+      }
     }
   } else if constexpr (EPI == EPI_LSE) {
     // per token of the chunk, (max, sum of exp(y - max)) over the tile's rows: 4 threads per token

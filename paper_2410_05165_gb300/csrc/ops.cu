@@ -3,6 +3,8 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <stdint.h>
+
 #include <algorithm>
 #include <cstring>
 #include <mutex>
@@ -83,7 +85,10 @@ atspeed_status atspeed_op_gemm(atspeed_stream stream, const void* d_W, const voi
 
 atspeed_status atspeed_op_gemm_swiglu(atspeed_stream stream, const void* d_W, const void* d_X, int F, int K, int T,
                                       int x_rows, void* d_out, int ldo, void* d_ws) {
-  if (!d_W || !d_X || !d_out || F <= 0 || K <= 0 || T <= 0 || ldo < F) return ATSPEED_E_ARG;
+  // the epilogue stores two adjacent bf16 outputs at once: ldo even, d_out 4-byte aligned
+  if (!d_W || !d_X || !d_out || F <= 0 || K <= 0 || T <= 0 || ldo < F || (ldo & 1) ||
+      (reinterpret_cast<uintptr_t>(d_out) & 3))
+    return ATSPEED_E_ARG;
   GemmArgs a = {};
   a.epi = EPI_SWIGLU;
   a.W = static_cast<const __nv_bfloat16*>(d_W);
