@@ -133,13 +133,15 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, in
                                           int ep_tid, const int* tpos, const int* tkvr) {
   const int tok0 = n_tile * BN + ch * 32;
   if constexpr (EPI == EPI_QKV) {
-    // rows of q | k | v.  Thread = (rotation pair, token parity): pair (i, i + hd/2) of one head
-    // shares its cos / sin, and the thread rotates both rows (rotate-half RoPE) for tokens
-    // (ep_tid >> 6) + 2k; k / v rows go to their cache rows, v rounded to bf16 and kept as fp16.
+    // rows of q | k | v.  Thread = (two adjacent rotation pairs, token quarter): pairs (i, i + hd/2)
+    // and (i + 1, i + 1 + hd/2) of one head (i even) for tokens (ep_tid >> 5) + 4k, so every load of
+    // the staged rows and the rotary tables and every store moves two adjacent values (rotate-half
+    // RoPE, the same arithmetic per element); k / v rows go to their cache rows, v rounded to bf16
+    // and kept as fp16.
     const int d = a.d_model, hd = a.head_dim, half = hd >> 1;
-    const int pi = ep_tid & 63, n0 = ep_tid >> 6;
+    const int pi = 2 * (ep_tid & 31), n0 = ep_tid >> 5;
     const int hh = pi / half, i = pi - hh * half;
-    const int r_lo = hh * hd + i, r_hi = r_lo + half;     // rows within the tile
+    const int r_lo = hh * hd + i, r_hi = r_lo + half;     // rows within the tile (r_lo even)
     const int row = m_tile * GEMM_BM + r_lo;
     if (row >= a.M) return;                                // padding rows of the last tile
     const int region = row / d;
@@ -148,33 +150,40 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, in
     const int tt0 = ch * 32;                               // token-table index of the chunk's first token
     if (region == 2) {
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const int n = n0 + 2 * k;
+      for (int k = 0; k < 8; ++k) {
+        const int n = n0 + 4 * k;
         if (n < nv) {
           __half* vr = a.v_cache + (size_t)tkvr[tt0 + n] * d;
-          vr[f_lo] = __float2half_rn(bf16_round(st[n * GEMM_BM + r_lo]));
-          vr[f_hi] = __float2half_rn(bf16_round(st[n * GEMM_BM + r_hi]));
+          const float2 lo = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_lo);
+          const float2 hi = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_hi);
+          *reinterpret_cast<__half2*>(vr + f_lo) =
+              __halves2half2(__float2half_rn(bf16_round(lo.x)), __float2half_rn(bf16_round(lo.y)));
+          *reinterpret_cast<__half2*>(vr + f_hi) =
+              __halves2half2(__float2half_rn(bf16_round(hi.x)), __float2half_rn(bf16_round(hi.y)));
         }
       }
     } else {
-      float cth[16], sth[16];
+      float2 cth[8], sth[8];
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const int n = n0 + 2 * k;
+      for (int k = 0; k < 8; ++k) {
+        const int n = n0 + 4 * k;
         const size_t cs = (size_t)tpos[tt0 + (n < nv ? n : 0)] * half + i;
-        cth[k] = a.rope_cos[cs];
-        sth[k] = a.rope_sin[cs];
+        cth[k] = *reinterpret_cast<const float2*>(a.rope_cos + cs);
+        sth[k] = *reinterpret_cast<const float2*>(a.rope_sin + cs);
       }
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const int n = n0 + 2 * k;
+      for (int k = 0; k < 8; ++k) {
+        const int n = n0 + 4 * k;
         if (n < nv) {
-          const float x_lo = st[n * GEMM_BM + r_lo], x_hi = st[n * GEMM_BM + r_hi];
-          const __nv_bfloat16 o_lo = __float2bfloat16_rn(x_lo * cth[k] - x_hi * sth[k]);
-          const __nv_bfloat16 o_hi = __float2bfloat16_rn(x_hi * cth[k] + x_lo * sth[k]);
+          const float2 xl = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_lo);
+          const float2 xh = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_hi);
+          const __nv_bfloat16 o_lo0 = __float2bfloat16_rn(xl.x * cth[k].x - xh.x * sth[k].x);
+          const __nv_bfloat16 o_hi0 = __float2bfloat16_rn(xh.x * cth[k].x + xl.x * sth[k].x);
+          const __nv_bfloat16 o_lo1 = __float2bfloat16_rn(xl.y * cth[k].y - xh.y * sth[k].y);
+          const __nv_bfloat16 o_hi1 = __float2bfloat16_rn(xh.y * cth[k].y + xl.y * sth[k].y);
           __nv_bfloat16* orow = region == 0 ? a.q_out + (size_t)(tok0 + n) * d : a.k_cache + (size_t)tkvr[tt0 + n] * d;
-          orow[f_lo] = o_lo;
-          orow[f_hi] = o_hi;
+          *reinterpret_cast<__nv_bfloat162*>(orow + f_lo) = __halves2bfloat162(o_lo0, o_lo1);
+          *reinterpret_cast<__nv_bfloat162*>(orow + f_hi) = __halves2bfloat162(o_hi0, o_hi1);
         }
       }
     }
