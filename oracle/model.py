@@ -76,14 +76,25 @@ def _layer_pre_attn(m: Model, l: int, h: np.ndarray, pos: np.ndarray):
     return q, k, v
 
 
-def _layer_post_attn(m: Model, l: int, h: np.ndarray, o: np.ndarray) -> np.ndarray:
+def _layer_mlp_act(m: Model, l: int, h: np.ndarray, o: np.ndarray):
+    """O projection added to the residual, RMSNorm, gate/up projection and the SwiGLU product.
+    Returns (residual after the attention block, rounded SwiGLU product)."""
     sp = m.spec
     f = sp.d_ffn
     h = h + m.rnd(o).reshape(h.shape[0], -1) @ m.W(f"layers.{l}.wo").T
     x2 = m.rnd(rmsnorm(h, m.W(f"layers.{l}.mlp_norm"), sp.rms_eps))
     gu = x2 @ m.W(f"layers.{l}.wgate_up").T
-    a = m.rnd(silu(gu[:, :f]) * gu[:, f:])
+    return h, m.rnd(silu(gu[:, :f]) * gu[:, f:])
+
+
+def _layer_mlp_out(m: Model, l: int, h: np.ndarray, a: np.ndarray) -> np.ndarray:
+    """Down projection of the SwiGLU product added to the residual."""
     return h + a @ m.W(f"layers.{l}.wdown").T
+
+
+def _layer_post_attn(m: Model, l: int, h: np.ndarray, o: np.ndarray) -> np.ndarray:
+    h, a = _layer_mlp_act(m, l, h, o)
+    return _layer_mlp_out(m, l, h, a)
 
 
 def _attend(q: np.ndarray, K: np.ndarray, V: np.ndarray, mask: Optional[np.ndarray]) -> np.ndarray:

@@ -91,6 +91,52 @@ def _philox_inverse(x, k0, k1):
     return y0, y1, y2, y3
 
 
+# An independent Philox4x32-10: the one in Triton's language library (tl.philox), run by Triton's
+# CPU interpreter in a child process (the interpreter is chosen by an environment variable read at
+# import).  It fixes the round multipliers, which the inversion test below cannot (it inverts with
+# the oracle's own multipliers), and the whole round and key schedule of Salmon et al. (SC'11).
+_TRITON_PHILOX = r"""
+import json, os, sys
+os.environ["TRITON_INTERPRET"] = "1"
+import torch, triton, triton.language as tl
+
+@triton.jit
+def kern(c_ptr, k_ptr, o_ptr, N: tl.constexpr):
+    i = tl.arange(0, N)
+    seed = (tl.load(k_ptr + 2 * i + 1).to(tl.uint64) << 32) | tl.load(k_ptr + 2 * i).to(tl.uint64)
+    r0, r1, r2, r3 = tl.philox(seed, tl.load(c_ptr + 4 * i), tl.load(c_ptr + 4 * i + 1),
+                               tl.load(c_ptr + 4 * i + 2), tl.load(c_ptr + 4 * i + 3), 10)
+    tl.store(o_ptr + 4 * i, r0)
+    tl.store(o_ptr + 4 * i + 1, r1)
+    tl.store(o_ptr + 4 * i + 2, r2)
+    tl.store(o_ptr + 4 * i + 3, r3)
+
+rows = json.load(sys.stdin)
+n = len(rows)
+c = torch.tensor([x for r in rows for x in r[:4]], dtype=torch.int64).to(torch.int32)
+k = torch.tensor([x for r in rows for x in r[4:]], dtype=torch.int64).to(torch.uint32)
+o = torch.zeros(4 * n, dtype=torch.int32)
+kern[(1,)](c, k, o, N=n)
+print(json.dumps([x & 0xFFFFFFFF for x in o.tolist()]))
+"""
+
+
+def test_philox_matches_triton_library():
+    import json
+    import subprocess
+    import sys
+    pytest.importorskip("triton")
+    rng = np.random.default_rng(17)
+    rows = [[0] * 6, [0xFFFFFFFF] * 6, [1, 2, 3, 4, 5, 6]]
+    rows += [[int(v) for v in rng.integers(0, 2 ** 32, size=6, dtype=np.uint64)] for _ in range(125)]
+    r = subprocess.run([sys.executable, "-c", _TRITON_PHILOX], input=json.dumps(rows), capture_output=True,
+                       text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lib = np.array(json.loads(r.stdout.strip().splitlines()[-1]), dtype=np.uint64).reshape(-1, 4)
+    ours = np.stack([np.array([int(x) for x in philox4x32_10(*row)], dtype=np.uint64) for row in rows])
+    np.testing.assert_array_equal(ours, lib)
+
+
 def test_philox_inverts_to_its_counter():
     rng = np.random.default_rng(5)
     for _ in range(200):
