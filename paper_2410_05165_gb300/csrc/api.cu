@@ -1746,6 +1746,20 @@ atspeed_status atspeed_debug_buffer(atspeed_ctx* c, int which, int id, void* h_o
       case 8: src = c->fwd_bar; cap = 4; break;
       case 9: src = c->fwd_trace; cap = c->fwd_trace_n * 8; break;
       case 10: src = m.lse; cap = (size_t)m.logit_rows * 4; break;
+      case 11: src = m.tok; cap = (size_t)m.Tcap * 4; break;
+      case 12: src = m.pos; cap = (size_t)m.Tcap * 4; break;
+      case 13: src = m.kvrow; cap = (size_t)m.Tcap * 4; break;
+      case 14: src = m.anc; cap = (size_t)m.Tcap * 16; break;
+      case 15: src = m.ancn; cap = (size_t)m.Tcap * 4; break;
+      case 16: {  // geometry, from the host
+        const int32_t g[4] = {m.rows, m.Tcap, m.Xrows, c->prefix_pages_per_user};
+        if (!m.present || !h_out || bytes > sizeof g) {
+          set_err(c, "debug_buffer: bad arguments");
+          throw Fail{ATSPEED_E_ARG};
+        }
+        memcpy(h_out, g, bytes);
+        return;
+      }
       default: break;
     }
     if (!m.present || !src || !h_out || bytes > cap) {
