@@ -197,8 +197,12 @@ atspeed_status atspeed_profile_read(atspeed_ctx *ctx, int kind, int32_t *h_launc
  * 6 V cache (fp16), 7 item-code logits (fp32 [rows][1024]), 8 the persistent forward's barrier
  * counter (u32), 9 its per-phase timestamps ([phases][CTAs] u64 ns, recorded only when the
  * environment variable ATSPEED_FWD_TRACE=1 was set at create time), 10 the whole-vocabulary
- * log-sum-exp of each logits row (fp32 [rows], written under FULL normalisation).
- * Synchronises the device. */
+ * log-sum-exp of each logits row (fp32 [rows], written under FULL normalisation); the last
+ * forward's per-token tables (int32 [T]): 11 token ids, 12 rotary positions, 13 K/V cache rows,
+ * 14 the cache rows of each token's path keys ([T][4]), 15 their count; 16 the buffer geometry
+ * (int32 [4]: K/V cache rows per layer, token capacity, allocated rows of x, prefix pages per
+ * user; user u's history token p sits in cache row u * 64 * pages + p).
+ * Synchronises the device (except id 16). */
 atspeed_status atspeed_debug_buffer(atspeed_ctx *ctx, int which, int id, void *h_out, size_t bytes);
 
 /* Shape of the current speculative step: h_depth[n_users], h_levels[n_users] (drafted levels),
@@ -239,7 +243,10 @@ atspeed_status atspeed_set_tree(atspeed_ctx *ctx, atspeed_stream stream, int n_l
 /* Y[t][m] = sum_k W[m][k] X[t][k] (+ Y when accumulate) with W bf16 [M][K], X bf16 [x_rows][K]
  * (x_rows >= T rounded up to 128, or to 256 when T > 128), Y fp32 [T][ldy].  tcgen05 tensor cores,
  * fp32 accumulation.  K must be a multiple of 64.  Needs atspeed_op_workspace_bytes() of d_ws
- * (zero-filled before its first use; every call leaves its counter part zeroed again). */
+ * (zero-filled before its first use; every call leaves its counter part zeroed again).  Returns
+ * ATSPEED_E_SHAPE for a shape it cannot run, ATSPEED_E_ARG for a null or misaligned operand (W, X
+ * need 16-byte aligned rows), ATSPEED_E_CUDA for a failed launch; device-side timeouts surface
+ * through atspeed_op_status. */
 size_t atspeed_op_workspace_bytes(void);
 atspeed_status atspeed_op_gemm(atspeed_stream stream, const void *d_W, const void *d_X, int M, int K, int T,
                                int x_rows, float *d_Y, int ldy, int accumulate, void *d_ws);
@@ -260,6 +267,17 @@ atspeed_status atspeed_op_gemm(atspeed_stream stream, const void *d_W, const voi
  * before any stream capture.  The paper has no counterpart: it is a deployment convenience. */
 atspeed_status atspeed_op_gemm_noalloc(atspeed_stream stream, const void *d_W, const void *d_X, int M, int K, int T,
                                        int x_rows, float *d_Y, int ldy, int accumulate);
+
+/* Device-side failures of the op GEMMs above (atspeed_op_gemm, atspeed_op_gemm_swiglu,
+ * atspeed_op_gemm_noalloc).  Their launches return ATSPEED_OK once enqueued; a bounded wait inside
+ * the kernel that gives up (a copy or a peer CTA that never arrives) does not trap but sets an error
+ * word in the call's scratch, which stays set (sticky) across later calls until this function reads
+ * it.  Synchronises `stream`, reads and clears the word of the workspace d_ws (or, with d_ws = NULL,
+ * of the allocation-free entry point's scratch on the current device) and returns ATSPEED_OK,
+ * ATSPEED_E_TIMEOUT (a bounded wait gave up: the outputs of the calls since the last check are not
+ * valid) or ATSPEED_E_CUDA (the synchronisation or the read failed).  Not part of the paper: it is
+ * how the stateless operators report device errors. */
+atspeed_status atspeed_op_status(atspeed_stream stream, void *d_ws);
 
 /* out[t][j] = bf16(silu(G[t][j]) * U[t][j]) with G = X W[0:F]^T, U = X W[F:2F]^T (SwiGLU), W bf16
  * [2F][K]; out bf16 [T][ldo] with ldo even and d_out 4-byte aligned (ATSPEED_E_ARG otherwise). */

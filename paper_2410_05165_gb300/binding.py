@@ -26,7 +26,7 @@ EXPORTS = [
     "atspeed_draft_step", "atspeed_verify", "atspeed_draft_step_logits", "atspeed_verify_logits",
     "atspeed_beam_search", "atspeed_set_early_reject", "atspeed_profile", "atspeed_profile_read", "atspeed_tree_shape", "atspeed_debug_tree",
     "atspeed_debug_node_logits", "atspeed_debug_node_lse", "atspeed_debug_buffer", "atspeed_set_tree", "atspeed_op_workspace_bytes", "atspeed_op_gemm",
-    "atspeed_op_gemm_noalloc", "atspeed_op_gemm_swiglu", "atspeed_op_rmsnorm", "atspeed_op_attention_scratch", "atspeed_op_attention",
+    "atspeed_op_gemm_noalloc", "atspeed_op_status", "atspeed_op_gemm_swiglu", "atspeed_op_rmsnorm", "atspeed_op_attention_scratch", "atspeed_op_attention",
 ]
 
 
@@ -100,6 +100,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "atspeed_op_gemm": (c_int, [vp, vp, vp, c_int, c_int, c_int, c_int, vp, c_int, c_int, vp]),
         "atspeed_op_gemm_noalloc": (c_int, [vp, vp, vp, c_int, c_int, c_int, c_int, vp, c_int, c_int]),
         "atspeed_op_gemm_swiglu": (c_int, [vp, vp, vp, c_int, c_int, c_int, c_int, vp, c_int, vp]),
+        "atspeed_op_status": (c_int, [vp, vp]),
         "atspeed_op_rmsnorm": (c_int, [vp, vp, vp, c_int, c_int, ctypes.c_float, vp, c_int]),
         "atspeed_op_attention_scratch": (ctypes.c_size_t, [c_int, c_int, c_int, c_int]),
         "atspeed_op_attention": (c_int, [vp, vp, vp, vp, c_int, c_int, c_int, c_int, c_int, i32p, i32p, i32p, i32p,
@@ -355,6 +356,13 @@ def op_gemm_noalloc(W: torch.Tensor, X: torch.Tensor, T: int, Y: Optional[torch.
     _check(load().atspeed_op_gemm_noalloc(_stream(stream), W.data_ptr(), X.data_ptr(), M, K, T, X.shape[0],
                                           Y.data_ptr(), Y.shape[1], 1 if accumulate else 0))
     return Y
+
+
+def op_status(noalloc: bool = False, stream=None) -> int:
+    """atspeed_op_status: synchronises, reads and clears the device error word of the op GEMMs'
+    workspace (or of the allocation-free scratch); returns the status code (0 = no device error)."""
+    ws = None if noalloc else op_workspace().data_ptr()
+    return int(load().atspeed_op_status(_stream(stream), ws))
 
 
 def op_gemm_swiglu(W: torch.Tensor, X: torch.Tensor, T: int, stream=None) -> torch.Tensor:

@@ -60,11 +60,10 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn_att() {
 template <int HD>
 cudaError_t launch_hd(const AttnArgs& a, const CUtensorMap& mk, const CUtensorMap& mv, cudaStream_t st, bool pdl) {
   using C = AttCfg<HD>;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(attn_prefix_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  static std::atomic<unsigned long long> attr_done{0};
+  {
+    const cudaError_t e = smem_attr_once(attr_done, attn_prefix_kernel<HD>, C::SMEM);
     if (e != cudaSuccess) return e;
-    attr = true;
   }
   cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -10,6 +10,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #define ATSPEED_DEV_ERR_TIMEOUT 1u
 #define ATSPEED_DEV_ERR_BOUNDS 2u
 
@@ -203,6 +205,20 @@ __device__ __forceinline__ bool named_bar_and(int id, int nthreads, bool v) {
       : "r"((uint32_t)v), "r"(id), "r"(nthreads)
       : "memory");
   return r != 0;
+}
+
+// Raises a kernel's dynamic shared-memory limit to `bytes` on the current device, once per device
+// (the attribute is per device; `done` holds one bit per device ordinal below 64).
+template <class Kern>
+inline cudaError_t smem_attr_once(std::atomic<unsigned long long>& done, Kern kernel, int bytes) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = dev < 64 ? (1ull << dev) : 0ull;
+  if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_acq_rel);
+  return e;
 }
 
 __device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }

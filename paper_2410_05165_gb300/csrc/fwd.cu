@@ -1014,11 +1014,10 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
 template <int HD, int BN>
 cudaError_t launch_t(const FwdParams& p, cudaStream_t st) {
   using LY = FLayout<HD, BN>;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(fwd_kernel<HD, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, LY::TOTAL);
+  static std::atomic<unsigned long long> attr_done{0};
+  {
+    const cudaError_t e = smem_attr_once(attr_done, fwd_kernel<HD, BN>, LY::TOTAL);
     if (e != cudaSuccess) return e;
-    attr = true;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.G);

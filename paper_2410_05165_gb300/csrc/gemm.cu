@@ -340,12 +340,9 @@ bool make_map(CUtensorMap* m, const void* base, int inner, int rows, int box_row
 template <int BN, int EPI>
 cudaError_t launch_t(const CUtensorMap& ma, const CUtensorMap& mb, const KParams& kp, cudaStream_t st, bool pdl) {
   using C = Cfg<BN>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static std::atomic<unsigned long long> attr_done{0};
+  const cudaError_t e = smem_attr_once(attr_done, gemm_kernel<BN, EPI>, C::SMEM);
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(kp.G);
   cfg.blockDim = dim3(192);
@@ -449,8 +446,9 @@ cudaError_t gemm_launch(const GemmArgs& a, const GemmScratch& s, int grid, cudaS
   kp.counters = s.counters;
   kp.err = s.err;
   CUtensorMap ma, mb;
-  if (!make_map(&ma, a.W, a.K, a.M, 64, eb, el)) return cudaErrorInvalidValue;
-  if (!make_map(&mb, a.X, a.K, a.X_rows, BN, eb, el)) return cudaErrorInvalidValue;
+  // an operand the tensor-map encoder refuses (typically a base address that is not 16-byte aligned)
+  if (!make_map(&ma, a.W, a.K, a.M, 64, eb, el)) return kGemmMapError;
+  if (!make_map(&mb, a.X, a.K, a.X_rows, BN, eb, el)) return kGemmMapError;
   return BN == 128 ? launch_bn<128>(a.epi, ma, mb, kp, stream, pdl) : launch_bn<256>(a.epi, ma, mb, kp, stream, pdl);
 }
 

@@ -62,6 +62,10 @@ int gemm_grid_size(int device);
 // 2D bf16 tensor map over a row-major [rows][inner] matrix, box {64, box_rows}, 128B swizzle.
 bool gemm_make_map(CUtensorMap* m, const void* base, int inner, int rows, int box_rows, char* eb, size_t el);
 
+// gemm_launch's return value when an operand cannot be described by a tensor map (its base
+// address or row pitch breaks the TMA alignment rules); cudaErrorInvalidValue means a bad shape.
+constexpr cudaError_t kGemmMapError = cudaErrorInvalidDevicePointer;
+
 // Encodes the tensor maps and launches.  `pdl` enables programmatic dependent launch.
 cudaError_t gemm_launch(const GemmArgs& a, const GemmScratch& s, int grid, cudaStream_t stream, bool pdl,
                         char* errbuf, size_t errlen);

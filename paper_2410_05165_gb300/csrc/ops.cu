@@ -13,6 +13,7 @@
 #include "atspeed.h"
 #include "attention.cuh"
 #include "gemm.cuh"
+#include "common.cuh"
 #include "kernels.cuh"
 
 using namespace atspeed;
@@ -36,12 +37,19 @@ GemmScratch scratch_from(void* ws) {
   return s;
 }
 
+// gemm_launch result -> status: a refused shape is E_SHAPE, an operand the tensor-map encoder
+// refuses (misaligned base address) is E_ARG, any other launch failure is E_CUDA.
+atspeed_status gemm_status(cudaError_t e) {
+  if (e == cudaSuccess) return ATSPEED_OK;
+  if (e == cudaErrorInvalidValue) return ATSPEED_E_SHAPE;
+  if (e == kGemmMapError) return ATSPEED_E_ARG;
+  return ATSPEED_E_CUDA;
+}
+
 atspeed_status run_gemm(cudaStream_t st, const GemmArgs& a, void* ws) {
   if (!ws) return ATSPEED_E_ARG;
   char eb[256];
-  const cudaError_t e = gemm_launch(a, scratch_from(ws), current_grid(), st, false, eb, sizeof eb);
-  if (e == cudaErrorInvalidValue) return ATSPEED_E_SHAPE;
-  return e == cudaSuccess ? ATSPEED_OK : ATSPEED_E_CUDA;
+  return gemm_status(gemm_launch(a, scratch_from(ws), current_grid(), st, false, eb, sizeof eb));
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -58,6 +66,23 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
 
 std::mutex g_noalloc_mu;
 void* g_noalloc_ptr[64] = {nullptr};
+
+// Device address of the allocation-free scratch on the current device, looked up on first use.
+void* noalloc_base() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return nullptr;
+    g_noalloc_ptr[dev] = ptr;
+  }
+  return g_noalloc_ptr[dev];
+}
+
+unsigned int* noalloc_err_word(void* base) {
+  return reinterpret_cast<unsigned int*>(static_cast<char*>(base) + kNoAllocWsBytes + (size_t)kNoAllocTiles * 4);
+}
 
 }  // namespace
 
@@ -215,25 +240,16 @@ atspeed_status atspeed_op_gemm_noalloc(atspeed_stream stream, const void* d_W, c
   const int BN = T <= 128 ? 128 : 256;
   const long long tiles = (long long)((M + 127) / 128) * ((T + BN - 1) / BN);
   if (tiles > kNoAllocTiles || K % 64 != 0 || K / 64 > 256) return ATSPEED_E_SHAPE;
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return ATSPEED_E_CUDA;
-  void* base = nullptr;
-  {
-    std::lock_guard<std::mutex> lk(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
-      void* ptr = nullptr;
-      if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return ATSPEED_E_CUDA;
-      g_noalloc_ptr[dev] = ptr;
-    }
-    base = g_noalloc_ptr[dev];
-  }
+  void* base = noalloc_base();
+  if (!base) return ATSPEED_E_CUDA;
   GemmScratch s;
   s.ws = static_cast<float*>(base);
   s.ws_bytes = kNoAllocWsBytes;
   s.counters = reinterpret_cast<int*>(static_cast<char*>(base) + kNoAllocWsBytes);
   s.max_tiles = kNoAllocTiles;
-  s.err = reinterpret_cast<unsigned int*>(static_cast<char*>(base) + kNoAllocWsBytes + (size_t)kNoAllocTiles * 4);
-  // the tile counters must start at zero (a call that failed part-way could have left some set)
+  s.err = noalloc_err_word(base);
+  // the tile counters must start at zero (a call that failed part-way could have left some set);
+  // the error word after them is left alone: it is sticky until atspeed_op_status reads it
   if (cudaMemsetAsync(s.counters, 0, (size_t)kNoAllocTiles * sizeof(int), (cudaStream_t)stream) != cudaSuccess)
     return ATSPEED_E_CUDA;
   GemmArgs a = {};
@@ -247,9 +263,26 @@ atspeed_status atspeed_op_gemm_noalloc(atspeed_stream stream, const void* d_W, c
   a.out_f32 = d_Y;
   a.ldo = ldy;
   char eb[256];
-  const cudaError_t e = gemm_launch(a, s, kNoAllocGrid, (cudaStream_t)stream, false, eb, sizeof eb);
-  if (e == cudaErrorInvalidValue) return ATSPEED_E_SHAPE;
-  return e == cudaSuccess ? ATSPEED_OK : ATSPEED_E_CUDA;
+  return gemm_status(gemm_launch(a, s, kNoAllocGrid, (cudaStream_t)stream, false, eb, sizeof eb));
+}
+
+/* See include/atspeed.h.  Reads (and clears) the error word that the op GEMMs' bounded waits set. */
+atspeed_status atspeed_op_status(atspeed_stream stream, void* d_ws) {
+  unsigned int* word = nullptr;
+  if (d_ws) {
+    word = scratch_from(d_ws).err;
+  } else {
+    void* base = noalloc_base();
+    if (!base) return ATSPEED_E_CUDA;
+    word = noalloc_err_word(base);
+  }
+  cudaStream_t st = (cudaStream_t)stream;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return ATSPEED_E_CUDA;
+  unsigned int v = 0;
+  if (cudaMemcpy(&v, word, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return ATSPEED_E_CUDA;
+  if (v == 0) return ATSPEED_OK;
+  if (cudaMemset(word, 0, sizeof v) != cudaSuccess) return ATSPEED_E_CUDA;
+  return (v & ATSPEED_DEV_ERR_TIMEOUT) ? ATSPEED_E_TIMEOUT : ATSPEED_E_CUDA;
 }
 
 }  // extern "C"
