@@ -90,8 +90,10 @@ def parse():
     return ap.parse_args()
 
 
-# DRAM bytes per algorithmic byte of the verification-call forward kernel, from the ncu capture in
-# profiles/fwd_kernel_verify_7b2l_full.md (863.9 MB of traffic for 838.7 MB of algorithmic bytes).
+# DRAM bytes per algorithmic byte of the batch-1 verification-call forward kernel (T = 120 tree
+# tokens): dram__bytes_read.sum + dram__bytes_write.sum of one ncu capture of the same kernel with
+# the target cut to 2 layers (863.9 MB of traffic for 838.7 MB of algorithmic bytes).  Measured for
+# the 128-token-tile schedule only: other workloads report no traffic figure.
 TRAFFIC_PER_ALG_BYTE = 863.9 / 838.7
 
 
@@ -342,20 +344,22 @@ def run_ours(args, w):
                 "peak_note": "sustained bf16 (a launch of several ms)"}
     roof["frac"] = roof["achieved"] / roof["peak"]
 
+    lo, hi = w.prompt_len
+    p_label = str(lo) if lo == hi else f"U[{lo},{hi}] (mean {np.mean(P_users):.0f})"
     line = {
         "metric": METRIC, "value": value, "unit": "rec lists/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights, synthetic items)",
         "config": {"workload": f"{w.name}: 7B-shape target (32L d4096 H32 ffn11008 V33024), draft 4L d768, "
-                               f"K={w.K} N={w.N} gamma={w.gamma}, P={w.prompt_len[0]}, {w.n_items} Zipf items, "
+                               f"K={w.K} N={w.N} gamma={w.gamma}, P={p_label}, {w.n_items} Zipf items, "
                                f"{args.mode} verification, {args.norm} normalisation, {B} user(s) per GPU"
                                + (", early rejection at depth 0" if args.early_reject else ""),
                    "l2": "inputs larger than L2 (13.5 GB of target weights per verification call)"},
         "roofline": dict(roof, **{
-            "traffic": TRAFFIC_PER_ALG_BYTE * vb,
-            "traffic_source": "dram__bytes_read.sum + dram__bytes_write.sum of one ncu capture of the same "
-                              "kernel with the target cut to 2 layers, scaled by algorithmic bytes "
-                              "(profiles/fwd_kernel_verify_7b2l_full.md)",
+            "traffic": TRAFFIC_PER_ALG_BYTE * vb if T_first <= 128 else None,
+            "traffic_source": ("dram__bytes_read.sum + dram__bytes_write.sum of one ncu capture of the same "
+                               "kernel with the target cut to 2 layers, scaled by algorithmic bytes"
+                               if T_first <= 128 else "not captured at this tree size"),
             "kernel": f"fwd_kernel: persistent forward of the verification call (tcgen05 GEMMs, tree attention, "
                       f"norms; T={T_first} tree tokens)",
             "peak_source": peak_kind, "launches": fk["launches"], "avg_launch_ms": k_ms,
