@@ -65,12 +65,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase with the given parity to complete.  Returns false on timeout.
+// The clock is read once every 256 polls (the timer is slow to read; try_wait itself suspends the
+// thread for a while).
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned int* err) {
   if (mbar_try_wait(bar, parity)) return true;
-  unsigned long long t0 = globaltimer_ns();
-  while (true) {
+  const unsigned long long t0 = globaltimer_ns();
+  for (unsigned it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (globaltimer_ns() - t0 > kWaitBudgetNs) {
+    if ((it & 255u) == 0u && globaltimer_ns() - t0 > kWaitBudgetNs) {
       set_error(err, ATSPEED_DEV_ERR_TIMEOUT);
       return false;
     }
@@ -97,6 +99,13 @@ __device__ __forceinline__ uint64_t policy_evict_last() {
 }
 
 // 2D tiled load: x = innermost coordinate (elements, must be 16-byte aligned), y = row.
+// Bulk prefetch of one tensor-map box into L2 (no destination, no completion to wait for).
+__device__ __forceinline__ void tma_prefetch_l2_2d(const CUtensorMap* map, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
                                             uint64_t policy) {
   asm volatile(
