@@ -186,16 +186,23 @@ def relaxed_verify(tree: Tree, L: int, K: int, target_rows: RowsFn, draft_rows: 
                 prev, prev_sp, prev_sq = list(drafted), Cp.score[dpos], Cq.score[dpos]
                 continue
             if d + g < L:
+                # every step passed, item not complete: K draws without replacement from p at the
+                # next level (a draw at the wrong level or a top-K fails
+                # test_oracle_relaxed_laws.py::test_all_accepted_draws_next_level_from_target)
                 C2 = expand(drafted, Cp.score[dpos], rows_p(drafted), trie)
                 keys = (C2.score + rng.gumbel(STREAM_RESAMPLE, lvl + 1, C2.index)).astype(F32)
                 sel = rank_order(keys, C2.index)[:K]
                 out, sp = _rank(child_paths(drafted, C2, sel), C2.score[sel], C2.index[sel])
                 return StepResult(g, g + 1, out, sp, len(acc))
+            # item complete: K picks uniform over the K-subsets of A (taking the first K of A fails
+            # test_oracle_relaxed_laws.py::test_complete_item_picks_uniform_subset_of_accepted)
             keys = rng.u32(STREAM_SUBSET, lvl, acc).astype(np.int64)
             pick = acc[np.lexsort((acc, keys))[:K]]
             out, sp = _rank([drafted[i] for i in pick], Cp.score[dpos[pick]], Cp.index[dpos[pick]])
             return StepResult(g, g, out, sp, len(acc))
         # step rejected: keep A, resample K - |A| from norm(max(0, p - q)) with p' = 0 on A
+        # (drawing from p or q instead, or letting A be drawn again, fails
+        # test_oracle_relaxed_laws.py::test_rejected_step_resamples_from_residual)
         p = np.exp(logp).astype(F32)
         q = np.exp(logq).astype(F32)
         pr = np.maximum(F32(0.0), (p - q).astype(F32))

@@ -99,13 +99,6 @@ __device__ __forceinline__ uint64_t policy_evict_last() {
 }
 
 // 2D tiled load: x = innermost coordinate (elements, must be 16-byte aligned), y = row.
-// Bulk prefetch of one tensor-map box into L2 (no destination, no completion to wait for).
-__device__ __forceinline__ void tma_prefetch_l2_2d(const CUtensorMap* map, int x, int y) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
-               "r"(x), "r"(y)
-               : "memory");
-}
-
 __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
                                             uint64_t policy) {
   asm volatile(
