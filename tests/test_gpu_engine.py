@@ -295,6 +295,51 @@ def test_sd_strict_lossless_and_matches_oracle_tiny(ats):
     ctx.close()
 
 
+# (history length, K, draft width N, gamma, items): a one-token history (one partly filled KV
+# page), histories ending at and just past a 64-row page, greedy K = 1, N = K, gamma = 1, a trie
+# with fewer items than K (every level keeps all its candidates, the list is padded), and the
+# largest gamma with the widest draft of the tiny limits
+EDGE_CASES = [(1, 5, 10, 2, 1000), (64, 3, 6, 3, 1000), (65, 4, 8, 2, 1000), (20, 1, 1, 1, 1000),
+              (33, 4, 4, 4, 1000), (12, 5, 10, 2, 3), (40, 2, 16, 4, 200)]
+
+
+@pytest.mark.parametrize("P,K,N,G,n_items", EDGE_CASES)
+def test_edge_cases_lossless_and_match_oracle(ats, P, K, N, G, n_items):
+    """Degenerate shapes end to end on the tiny models: SD strict == plain target beam search bit
+    for bit, and every returned item (and the padding when the trie has fewer than K items) against
+    the oracle's plain beam search on the same prompt."""
+    w = synth.workload("tiny")
+    items = synth.make_items(n_items, w.code_dist, w.zipf_a, w.seed + P)
+    prompt = synth.make_prompts(1, (P, P), w.target.vocab, w.seed + P)[0]
+    ctx = _ctx(ats, w.target, w.draft, items, w.code_base, 1, P, K, N, G, seed=w.seed)
+    toks = torch.from_numpy(prompt).cuda()
+    o = ats.opts(K, N, G)
+    sd_items, sd_sc, stats = ctx.beam_search(toks, [0, P], o, ats.SD_STRICT)
+    pl_items, pl_sc, _ = ctx.beam_search(toks, [0, P], o, ats.PLAIN_TOPK)
+    np.testing.assert_array_equal(sd_items.cpu().numpy(), pl_items.cpu().numpy())
+    np.testing.assert_array_equal(sd_sc.cpu().numpy(), pl_sc.cpu().numpy())
+    assert 1 <= stats[0, 1] <= L
+    tw = synth.model_weights(w.target, w.seed, "target")
+    trie = Trie(items)
+    ev = PathEvaluator(Model(w.target, tw, w.code_base), prompt)
+    item_rows = lambda ps: [ev.logits([p])[0][256 * len(p):256 * (len(p) + 1)].astype(np.float32) for p in ps]
+    ref, _ = plain_beam_search(item_rows, trie, K)
+    rows = sd_items[0].cpu().numpy()
+    sc = sd_sc[0].cpu().numpy()
+    got = [tuple(int(c) for c in r) for r in rows if r[0] >= 0]
+    n_valid = min(K, len(items))
+    assert len(got) == len(ref) == n_valid
+    assert np.all(rows[n_valid:] == -1) and np.all(np.isneginf(sc[n_valid:]))
+    assert len(set(got)) == n_valid and all(tuple(it) in set(map(tuple, items.tolist())) for it in got)
+    tol = 4 * 2e-2
+    osc = [_oracle_item_score(item_rows, trie, it) for it in got]
+    for it, g, r in zip(got, sc[:n_valid], osc):
+        assert abs(float(g) - r) < tol, (it, g, r)
+    if set(got) != set(ref):
+        assert _near_tie_level(item_rows, None, trie, K, tol), (got, ref)
+    ctx.close()
+
+
 def _oracle_item_score(item_rows, trie, it):
     """The oracle's masked sequence score of item `it` (fp64 sum of its L log-probs)."""
     import scipy.special
