@@ -32,6 +32,15 @@ namespace {
 constexpr int FWD_THREADS = 384;   // warps 0-3: producers, MMA (3 idle); warps 4-11: two compute warpgroups
 constexpr int COMPUTE_WARP0 = 4;
 constexpr int CT = 256;            // compute threads (named barrier 1); warpgroup w uses barrier 2 + w
+// Registers per thread after the prologue: the launch gives every thread 168 (12 warps, 3 per
+// SM sub-partition); warpgroup 0 (producers, MMA issuer, prefetch: little live state) gives back
+// down to kRegsRoles and the two compute warpgroups take them up to kRegsCompute, so that the
+// epilogues, norms and attention do not spill.  Budget (checked below): 128 * kRegsRoles + 256 *
+// kRegsCompute <= 384 * 168, and per sub-partition one role warp and two compute warps.
+constexpr int kRegsLaunch = 168, kRegsRoles = 80, kRegsCompute = 208;
+static_assert(128 * kRegsRoles + 256 * kRegsCompute <= FWD_THREADS * kRegsLaunch, "register split over the launch's total");
+static_assert(32 * (kRegsRoles + 2 * kRegsCompute) <= 16384, "register split over a sub-partition's file");
+static_assert(kRegsRoles % 8 == 0 && kRegsCompute % 8 == 0 && kRegsRoles >= 24 && kRegsCompute <= 256, "setmaxnreg range");
 constexpr int ITEM_ROWS_FWD = 1024;   // item-code rows of the LM head (4 levels x 256 codes)
 
 template <int BN>
@@ -774,7 +783,11 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-
+  // Each warpgroup sets its register count at the top of its own branch (every thread executes
+  // it; the compute warpgroups' request waits for the roles' release if it comes first), so that
+  // the code of each branch is allocated against its own count.
+  if (warp < COMPUTE_WARP0) {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsRoles));
   if (warp == 0) {
     // ------------------------------------------------------------- weight producer (never waits for the grid)
     if (lane == 0) {
@@ -903,7 +916,9 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
       tc_commit(mma_done);
       mbar_wait(mma_done, (uint32_t)(mma_waits & 1), nullptr);
     }
-  } else if (warp >= COMPUTE_WARP0) {
+  }
+  } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsCompute));
     // ------------------------------------------------------------- compute warps (two warpgroups)
     const int ctid = threadIdx.x - COMPUTE_WARP0 * 32;
     const int wg = ctid >> 7, wt = ctid & 127;
