@@ -164,6 +164,20 @@ __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* a) {
   return v;
 }
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Bulk (non-tensor) copy of `bytes` (a multiple of 16, both addresses 16-byte aligned) from this
+// CTA's shared memory to global memory, in its own bulk group.
+__device__ __forceinline__ void bulk_store(void* gdst, const void* ssrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\ncp.async.bulk.commit_group;" ::"l"(
+                   reinterpret_cast<uint64_t>(gdst)),
+               "r"(smem_u32(ssrc)), "r"(bytes)
+               : "memory");
+}
+// this thread's bulk stores have finished reading shared memory / are complete in global memory
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_done() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 __device__ __forceinline__ bool err_set(const unsigned* e) { return *(volatile const unsigned*)e != 0u; }
 
 // Waits until barrier `k` (0-based) is complete: count >= (k + 1) * G.  False on timeout or when an
@@ -545,6 +559,15 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       part_slot[pi] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
     }
   };
+  // a bulk copy of a split part (O / down projections) must have finished, in global memory and
+  // before its staging buffer is reused, when the phase ends (the next phases read the part with
+  // generic loads after the grid barrier, hence the proxy fence)
+  auto drain = [&]() {
+    if (wt == 0) {
+      bulk_wait_done();
+      fence_proxy_async();
+    }
+  };
   const bool shared_sums =
       !g.to_dh && (g.w.q > 0 || g.dh_out || (gi == 4 * p.L && g.w.Gsk > 0 && g.w.Usk / g.w.Gsk + 1 < kb));
   if (shared_sums && it.u < it.u1) {
@@ -554,7 +577,7 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       const int acc = si & 1, use = si >> 1;
       ++si;
       const bool got = named_bar_and(1, CT, mwait(&tfull[acc], (uint32_t)(use & 1), p.err));
-      if (!got) return false;
+      if (!got) { drain(); return false; }
       tc_fence_after();
       const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       const int nch = min(BN / 32, (g.rows - (tile % g.n_tiles) * BN + 31) / 32);
@@ -578,7 +601,7 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
       if (g.epi == EPI_QKV) load_tok_tables<BN>(ea, n_tile, tpos, tkvr, ctid, CT);
       if (ctid == 0) *flag = counter_wait(&skc[t], parts, p.err) ? 1 : 0;
       named_bar_sync(1, CT);
-      if (!*flag) return false;
+      if (!*flag) { drain(); return false; }
       const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
       int k = 0;
       for (int ch = c - c_first; ch < nch; ch += parts, ++k) {
@@ -609,12 +632,34 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
     }
     // (the vote is also the barrier after which token tables and part slots are in place)
     const bool got = named_bar_and(1, CT, mwait(&tfull[acc], (uint32_t)(use & 1), p.err));
-    if (!got) return false;
+    if (!got) { drain(); return false; }
     tc_fence_after();
     if (p.trace && ctid == 0) p.trace[((size_t)4 * NP + ph) * G + c] = globaltimer_ns();
     const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
     const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
     const int row = m_tile * GEMM_BM + m;
+    if (g.to_dh && !whole) {
+      // split part, [token][128 rows] fp32 in this CTA's workspace slot, where a 32-token chunk is
+      // 16 KB in one piece: TMEM -> the warpgroup's staging buffer -> one bulk copy per chunk
+      // (issued by one thread; the staging buffer is reused once that copy has read it)
+      float* slot = p.ws + ((long long)c * 2 + (seg == 0 ? 0 : 1)) * GEMM_WS_SLOT_FLOATS;
+      for (int ch = wg; ch < nch; ch += 2) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tb + ch * 32, r);
+        tmem_ld_wait();
+        const int nv = min(32, g.rows - n_tile * BN - ch * 32);
+        if (wt == 0) bulk_wait_read();
+        named_bar_sync(wbar, 128);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = __uint_as_float(r[j]);
+        fence_proxy_async_smem();   // the generic stores before the bulk copy's async reads
+        named_bar_sync(wbar, 128);
+        if (wt == 0) bulk_store(slot + (size_t)ch * 32 * GEMM_BM, staging, (uint32_t)nv * GEMM_BM * 4);
+      }
+      tc_fence_before();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      continue;
+    }
     if (g.to_dh) {
       float* dst;
       size_t ld;
@@ -708,6 +753,7 @@ __device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, 
     }
     named_bar_sync(1, CT);  // flag and part_slot are reused by the next segment
   }
+  drain();
   return true;
 }
 
