@@ -535,7 +535,7 @@ __device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* a
 // Parts are always summed in k order starting from zero, whichever CTA sums them.  Kept out of
 // line so that the epilogue gets its own register allocation.
 template <int BN>
-__device__ __noinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, float* staging_base, uint64_t* tfull,
+__device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, float* staging_base, uint64_t* tfull,
                                             uint64_t* tempty, int* flag, int* part_slot, int* tpos, int* tkvr,
                                             GemmArgs* s_ea, uint32_t tmem_base, int ctid, int& si) {
   const int c = blockIdx.x, G = p.G, NP = 7 * p.L + 2;
