@@ -187,7 +187,7 @@ __device__ bool grid_wait(const FwdParams& p, int k) {
   if (ld_acquire_u32(p.bar) >= target) return true;
   const unsigned long long t0 = globaltimer_ns();
   for (unsigned it = 1;; ++it) {
-    __nanosleep(64);
+    if (it > 32u) __nanosleep(64);   // back-to-back polls first: the barrier usually completes soon
     if (ld_acquire_u32(p.bar) >= target) return true;
     if ((it & 255u) == 0u) {
       if (err_set(p.err)) return false;
@@ -229,7 +229,7 @@ __device__ bool counter_wait(const int* cnt, int target, unsigned* err) {
   if ((int)ld_acquire_u32(reinterpret_cast<const unsigned*>(cnt)) >= target) return true;
   const unsigned long long t0 = globaltimer_ns();
   for (unsigned it = 1;; ++it) {
-    __nanosleep(64);
+    if (it > 32u) __nanosleep(64);
     if ((int)ld_acquire_u32(reinterpret_cast<const unsigned*>(cnt)) >= target) return true;
     if ((it & 255u) == 0u) {
       if (err_set(err)) return false;
