@@ -12,8 +12,12 @@ constexpr int GEMM_WS_SLOT_FLOATS = 256 * 128;
 // ---- work split of a tiled GEMM over G CTAs (tiles of kb k-blocks)
 // Each CTA takes q = tiles / G whole tiles; the first r = tiles % G tiles are split by k-blocks into
 // G equal contiguous unit ranges (stream-K; unit = one tile's k-block).  A CTA works on its
-// stream-K units first and then on its whole tiles r + c q ... r + c q + q - 1, so the partial sums
-// of the split tiles are published early and the tail after the last MMA is whole-tile epilogues.
+// stream-K units first and then on its whole tiles r + c, r + c + G, ..., r + c + (q - 1) G, so the
+// partial sums of the split tiles are published early and the tail after the last MMA is
+// whole-tile epilogues.  Whole tiles go round robin: at each step the grid works on G consecutive
+// tiles, i.e. (the token-tile index varying fastest) on every token tile of a few weight row tiles,
+// so each weight tile is read from DRAM about once per step and shared through L2 by the CTAs
+// that need it, where a contiguous range per CTA would have one CTA read it once per token tile.
 // With tiles < G (q = 0) this is plain stream-K over all tiles.
 struct WorkSplit {
   int tiles, kb, q, r;
@@ -75,7 +79,7 @@ __device__ __forceinline__ void cta_unit(const WorkSplit& w, int c, long long i,
   } else {
     const long long j = i - (b - a);
     const int t = (int)(j / w.kb);
-    tile = w.r + c * w.q + t;
+    tile = w.r + t * w.G + c;
     kbi = (int)(j - (long long)t * w.kb);
   }
 }
@@ -90,8 +94,8 @@ struct SegIter {
       return;
     }
     sk_range(w, c, u, u1);
-    dp = w.r + c * w.q;
-    dp1 = dp + w.q;
+    dp = w.r + c;                // whole tiles r + c, r + c + G, ... (round robin)
+    dp1 = w.r + w.q * w.G + c;
   }
   __device__ __forceinline__ bool next(const WorkSplit& w, int& tile, int& k0, int& k1) {
     if (u < u1) {
@@ -103,7 +107,8 @@ struct SegIter {
       return true;
     }
     if (dp < dp1) {
-      tile = dp++;
+      tile = dp;
+      dp += w.G;
       k0 = 0;
       k1 = w.kb;
       return true;
