@@ -192,7 +192,9 @@ atspeed_status atspeed_profile_read(atspeed_ctx *ctx, int kind, int32_t *h_launc
                                     double *h_flops);
 
 /* Copies the first `bytes` of one internal buffer of the target (which = 0) or draft (1) decoder
- * to the host: id 0 residual stream h (fp32 [T][d]), 1 normalised rows x (bf16), 2 q (bf16),
+ * to the host: id 0 residual stream h (fp32 [T][d]), 1 GEMM input rows x (bf16 [T][d]: the final
+ * norm's rows after a forward; during it, the gain-scaled residual g * h that feeds the QKV and
+ * gate/up projections, whose epilogues apply the norm's per-token scale), 2 q (bf16),
  * 3 attention output (bf16), 4 SwiGLU output (bf16 [T][d_ffn]), 5 K cache (bf16, all layers),
  * 6 V cache (fp16), 7 item-code logits (fp32 [rows][1024]), 8 the persistent forward's barrier
  * counter (u32), 9 its per-phase timestamps ([phases][CTAs] u64 ns, recorded only when the

@@ -7,7 +7,13 @@ attention -> O projection -> residual; RMSNorm -> SiLU-gated MLP -> residual.
 bf16 rounding points (both the oracle and the CUDA path round here, ties to
 even; everything else is fp64 here and fp32 on the GPU):
   * the embedding row (weights are bf16 already) enters an fp32/fp64 residual;
-  * RMSNorm outputs (the GEMM inputs);
+  * the inputs of the QKV and gate/up projections: RMSNorm(h) = s(h) * (g * h)
+    with the per-row scale s(h) = 1 / sqrt(mean(h^2) + eps), and since s(h)
+    is one number per token it commutes with the projection:
+    W RMSNorm(h) = s(h) * (W (g * h)).  The GEMM input is g * h, rounded to
+    bf16; s(h) multiplies the GEMM's output;
+  * the final RMSNorm's output (the LM head's input), rounded after the
+    whole norm;
   * q and k after RoPE, and v (k and v are stored as bf16 in the KV cache);
   * the attention output o (input of the O projection);
   * the SwiGLU product silu(gate) * up (input of the down projection).
@@ -27,7 +33,7 @@ from typing import Dict, List, Optional, Sequence, Tuple
 
 import numpy as np
 
-from .numerics import bf16, rmsnorm, rope, silu, softmax
+from .numerics import bf16, rms_scale, rmsnorm, rope, silu, softmax
 
 L_ITEM = 4
 CODES = 256
@@ -65,8 +71,8 @@ class Model:
 def _layer_pre_attn(m: Model, l: int, h: np.ndarray, pos: np.ndarray):
     sp = m.spec
     H, hd, d = sp.n_heads, sp.head_dim, sp.d_model
-    x = m.rnd(rmsnorm(h, m.W(f"layers.{l}.attn_norm"), sp.rms_eps))
-    qkv = x @ m.W(f"layers.{l}.wqkv").T
+    xg = m.rnd(h * m.W(f"layers.{l}.attn_norm"))
+    qkv = (xg @ m.W(f"layers.{l}.wqkv").T) * rms_scale(h, sp.rms_eps)
     q = qkv[:, :d].reshape(-1, H, hd)
     k = qkv[:, d:2 * d].reshape(-1, H, hd)
     v = qkv[:, 2 * d:].reshape(-1, H, hd)
@@ -77,13 +83,14 @@ def _layer_pre_attn(m: Model, l: int, h: np.ndarray, pos: np.ndarray):
 
 
 def _layer_mlp_act(m: Model, l: int, h: np.ndarray, o: np.ndarray):
-    """O projection added to the residual, RMSNorm, gate/up projection and the SwiGLU product.
+    """O projection added to the residual, RMSNorm, gate/up projection and the SwiGLU product
+    (the norm's scale applied to the projection's output, as in _layer_pre_attn).
     Returns (residual after the attention block, rounded SwiGLU product)."""
     sp = m.spec
     f = sp.d_ffn
     h = h + m.rnd(o).reshape(h.shape[0], -1) @ m.W(f"layers.{l}.wo").T
-    x2 = m.rnd(rmsnorm(h, m.W(f"layers.{l}.mlp_norm"), sp.rms_eps))
-    gu = x2 @ m.W(f"layers.{l}.wgate_up").T
+    x2g = m.rnd(h * m.W(f"layers.{l}.mlp_norm"))
+    gu = (x2g @ m.W(f"layers.{l}.wgate_up").T) * rms_scale(h, sp.rms_eps)
     return h, m.rnd(silu(gu[:, :f]) * gu[:, f:])
 
 

@@ -20,6 +20,12 @@ def bf16(x) -> np.ndarray:
     return np.ldexp(np.rint(m * 256.0), e - 8)
 
 
+def rms_scale(h: np.ndarray, eps: float) -> np.ndarray:
+    """RMSNorm's per-row scale 1 / sqrt(mean(h^2) + eps) over the last axis (keepdims)."""
+    h = np.asarray(h, dtype=np.float64)
+    return 1.0 / np.sqrt(np.mean(h * h, axis=-1, keepdims=True) + eps)
+
+
 def rmsnorm(h: np.ndarray, g: np.ndarray, eps: float) -> np.ndarray:
     """h / sqrt(mean(h^2) + eps) * g over the last axis."""
     h = np.asarray(h, dtype=np.float64)

@@ -78,7 +78,8 @@ struct ModelRt {
   // activations
   int Tcap = 0, Xrows = 0;
   float* h = nullptr;
-  float* dh = nullptr;   // persistent forward: product of the last O / down projection
+  float* ssq = nullptr;  // [ceil(d / 128)][Tcap] partial sums of squares of the residual rows per
+                         // 128-row tile (RMSNorm folded into the GEMMs around it)
   bf16 *x = nullptr, *q = nullptr, *att = nullptr, *act = nullptr;
   float* logits = nullptr;  // [logit_rows][1024]
   int logit_rows = 0;
@@ -390,7 +391,7 @@ void alloc_model(atspeed_ctx* c, ModelRt& m) {
   m.Tcap = std::max(L.max_users * L.max_prompt, L.max_users * stride);
   m.Xrows = ((m.Tcap + 255) / 256) * 256;
   m.h = dalloc<float>(c, (size_t)m.Tcap * m.d);
-  m.dh = dalloc<float>(c, (size_t)m.Tcap * m.d);
+  m.ssq = dalloc<float>(c, (size_t)((m.d + 127) / 128) * m.Tcap);
   m.x = dalloc<bf16>(c, (size_t)m.Xrows * m.d);
   m.q = dalloc<bf16>(c, (size_t)m.Tcap * m.d);
   m.att = dalloc<bf16>(c, (size_t)m.Xrows * m.d);
@@ -606,6 +607,7 @@ void gemm(atspeed_ctx* c, const GemmArgs& a, cudaStream_t st, int kind, int grid
   char eb[256] = {0};
   // algorithmic bytes: weights once, activations in, outputs out
   const double out_b = a.epi == EPI_F32 ? 4.0 * a.M : a.epi == EPI_RESID ? 8.0 * a.M
+                       : a.epi == EPI_RESNORM ? (a.gain ? 10.0 * a.M : 8.0 * a.M)
                        : a.epi == EPI_SWIGLU ? 1.0 * a.M : 2.0 * a.M;
   ProfScope ps(c, st, kind, 2.0 * a.M * a.K + 2.0 * a.T * a.K + out_b * a.T, 2.0 * a.M * a.K * a.T);
   cudaError_t e = gemm_launch(a, c->gs, grid, st, c->pdl && !c->prof, eb, sizeof eb);
@@ -673,7 +675,8 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     f.final_norm = m.final_norm;
     f.embed = m.embed;
     f.h = m.h;
-    f.dh = m.dh;
+    f.ssq = m.ssq;
+    f.ssq_ld = m.Tcap;
     f.x = m.x;
     f.q = m.q;
     f.att = m.att;
@@ -730,11 +733,19 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     c->n_launch += 1;
     return;
   }
+  // RMSNorm folded into the GEMMs: the O / down epilogues leave h, bf16(g * h) and per-tile sums of
+  // squares; the QKV / gate-up epilogues apply each token's 1 / rms
+  CK(embed_rows_launch(p.d_tokens, m.embed, m.attn_norm[0], m.h, m.x, m.ssq, m.Tcap, T, m.d, st, pdl));
+  c->n_launch += 1;
+  auto folded = [&](GemmArgs& g) {
+    g.ssq_ld = m.Tcap;
+    g.nrm_d = m.d;
+    g.eps = m.eps;
+  };
   for (int l = 0; l < m.layers; ++l) {
-    CK(rmsnorm_launch(m.h, l == 0 ? p.d_tokens : nullptr, m.embed, m.h, m.attn_norm[l], T, m.d, m.eps, m.x, m.d, st,
-                      pdl));
-    c->n_launch += 1;
     GemmArgs g = {};
+    folded(g);
+    g.ssq_in = m.ssq;
     g.epi = EPI_QKV;
     g.W = m.wqkv[l];
     g.X = m.x;
@@ -786,7 +797,11 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
       ps.done();
     }
     g = GemmArgs{};
-    g.epi = EPI_RESID;
+    folded(g);
+    g.epi = EPI_RESNORM;
+    g.gain = m.mlp_norm[l];
+    g.xg_out = m.x;
+    g.ssq_out = m.ssq;
     g.W = m.wo[l];
     g.X = m.att;
     g.M = m.d;
@@ -796,9 +811,9 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.out_f32 = m.h;
     g.ldo = m.d;
     gemm(c, g, st, 1, m.grid);
-    CK(rmsnorm_launch(m.h, nullptr, nullptr, nullptr, m.mlp_norm[l], T, m.d, m.eps, m.x, m.d, st, pdl));
-    c->n_launch += 1;
     g = GemmArgs{};
+    folded(g);
+    g.ssq_in = m.ssq;
     g.epi = EPI_SWIGLU;
     g.W = m.wgate_up[l];
     g.X = m.x;
@@ -810,7 +825,13 @@ void forward(atspeed_ctx* c, ModelRt& m, const FwdPlan& p, cudaStream_t st) {
     g.ldo = m.ffn;
     gemm(c, g, st, 2, m.grid);
     g = GemmArgs{};
-    g.epi = EPI_RESID;
+    folded(g);
+    g.epi = EPI_RESNORM;
+    if (l + 1 < m.layers) {   // (the final norm normalises the selected rows from h itself)
+      g.gain = m.attn_norm[l + 1];
+      g.xg_out = m.x;
+      g.ssq_out = m.ssq;
+    }
     g.W = m.wdown[l];
     g.X = m.act;
     g.M = m.d;

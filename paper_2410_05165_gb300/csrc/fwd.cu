@@ -1,8 +1,12 @@
 // Persistent forward kernel for sm_103a.
 //
 // One cooperative launch, one CTA per SM, runs a whole decoder forward as a fixed phase program:
-//   NORM0 | for each layer: QKV, ATTN, O, NORM, GATE_UP, DOWN, NORM | LM
-// with a grid barrier after every phase.  The GEMM phases reuse the stream-K decomposition of the
+//   EMBED | for each layer: QKV, ATTN, O, GATE_UP, DOWN | final NORM | LM
+// with a grid barrier after every phase.  The RMSNorms before the QKV and gate/up projections are
+// folded into the GEMMs around them (x = h / rms(h) * g, and W x = (W (g h)) / rms(h)): the O /
+// down epilogue adds its product to h and leaves bf16(g h) and per-128-row-tile sums of squares of
+// h; the QKV / gate-up epilogue multiplies each token's product by 1 / rms(h) from those sums.  (The
+// program keeps the index slots of the two norm phases per layer, 7 per layer, for the trace.)  The GEMM phases reuse the stream-K decomposition of the
 // standalone GEMM (equal contiguous ranges of (tile, k-block) units per CTA, split tiles reduced
 // by their last CTA), but their operands flow through two rings that live for the whole launch:
 //   * the weight ring (A, 16 KB per stage) is filled by a producer warp that walks every GEMM
@@ -74,10 +78,8 @@ struct FLayout {
 
 struct GP {
   int epi;
-  bool dh_out;   // O / down projection: the product goes to dh (the next norm phase adds it to h)
-  bool to_dh;    // ... with its split tiles' parts left in the workspace for the norm phase to sum
-                 // (few rows, BN = 128); with BN = 256 (many rows per CTA in the norm) the GEMM
-                 // phase sums them itself
+  int k;         // 0 QKV, 1 O, 2 gate/up, 3 down (of layer `layer`), 4 LM head
+  bool dh_out;   // O / down projection: the product is added to h (EPI_RESNORM)
   int M, K, m_tiles, n_tiles, kb, up_row0, rows;  // rows: valid tokens of the phase
   WorkSplit w;   // whole tiles per CTA + stream-K over the remaining tiles
   int mapA, mapB, layer;
@@ -91,8 +93,8 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
   g.up_row0 = 0;
   g.rows = p.T;
   g.dh_out = false;
-  g.to_dh = false;
   if (gi == 4 * L) {
+    g.k = 4;
     g.epi = EPI_F32;
     g.M = ITEM_ROWS_FWD;
     g.K = p.d;
@@ -101,6 +103,7 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
     g.rows = p.n_out;
   } else {
     const int k = gi % 4;
+    g.k = k;
     g.mapA = g.layer * 4 + k;
     if (k == 0) {
       g.epi = EPI_QKV;
@@ -108,9 +111,8 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
       g.K = p.d;
       g.mapB = act0;
     } else if (k == 1) {
-      g.epi = EPI_F32;
+      g.epi = EPI_RESNORM;
       g.dh_out = true;
-      g.to_dh = BN == 128;
       g.M = p.d;
       g.K = p.d;
       g.mapB = act0 + 1;
@@ -121,9 +123,8 @@ __device__ __forceinline__ GP gemm_phase(const FwdParams& p, int gi, int BN) {
       g.up_row0 = p.ffn;
       g.mapB = act0;
     } else {
-      g.epi = EPI_F32;
+      g.epi = EPI_RESNORM;
       g.dh_out = true;
-      g.to_dh = BN == 128;
       g.M = p.d;
       g.K = p.ffn;
       g.mapB = act0 + 2;
@@ -150,33 +151,12 @@ __device__ __forceinline__ void a_coords(const GP& g, int tile, int kbi, int& x,
   }
 }
 
-// phase index (in the compute warps' program) of GEMM phase gi
-__device__ __forceinline__ int gemm_phase_index(int gi, int L) {
-  if (gi == 4 * L) return 1 + 7 * L;
-  const int l = gi / 4, k = gi % 4;
-  return 7 * l + (k == 0 ? 1 : k == 1 ? 3 : k == 2 ? 5 : 6);
-}
-
-
 __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* a) {
   unsigned v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(a) : "memory");
   return v;
 }
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
-__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-
-// Bulk (non-tensor) copy of `bytes` (a multiple of 16, both addresses 16-byte aligned) from this
-// CTA's shared memory to global memory, in its own bulk group.
-__device__ __forceinline__ void bulk_store(void* gdst, const void* ssrc, uint32_t bytes) {
-  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\ncp.async.bulk.commit_group;" ::"l"(
-                   reinterpret_cast<uint64_t>(gdst)),
-               "r"(smem_u32(ssrc)), "r"(bytes)
-               : "memory");
-}
-// this thread's bulk stores have finished reading shared memory / are complete in global memory
-__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_done() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 __device__ __forceinline__ bool err_set(const unsigned* e) { return *(volatile const unsigned*)e != 0u; }
 
@@ -257,13 +237,15 @@ __device__ bool mwait(uint64_t* bar, uint32_t parity, unsigned* err) {
   }
 }
 
+// trs: the n-tile's norm scales (QKV / gate-up); bar: the warpgroup's named barrier (EPI_RESNORM)
 template <int BN>
-__device__ __noinline__ void epi_dispatch(int epi, const GemmArgs* a, const float* st, int mt, int nt, int ch,
-                                             int t, const int* tpos, const int* tkvr) {
+__device__ __noinline__ void epi_dispatch(int epi, const GemmArgs* a, float* st, int mt, int nt, int ch, int t,
+                                          const int* tpos, const int* tkvr, const float* trs, int bar) {
   switch (epi) {
     case EPI_F32: epi_chunk<BN, EPI_F32>(*a, st, mt, nt, ch, t, tpos, tkvr); break;
-    case EPI_SWIGLU: epi_chunk<BN, EPI_SWIGLU>(*a, st, mt, nt, ch, t, tpos, tkvr); break;
-    default: epi_chunk<BN, EPI_QKV>(*a, st, mt, nt, ch, t, tpos, tkvr); break;
+    case EPI_RESNORM: epi_resnorm(*a, st, mt, nt * BN + ch * 32, t, bar); break;
+    case EPI_SWIGLU: epi_chunk<BN, EPI_SWIGLU>(*a, st, mt, nt, ch, t, tpos, tkvr, trs); break;
+    default: epi_chunk<BN, EPI_QKV>(*a, st, mt, nt, ch, t, tpos, tkvr, trs); break;
   }
 }
 
@@ -282,9 +264,21 @@ __device__ GemmArgs epi_args(const FwdParams& p, const GP& g) {
   a.q_out = p.q;
   a.k_cache = p.kc + p.layer_elems * g.layer;
   a.v_cache = p.vc + p.layer_elems * g.layer;
+  a.ssq_ld = p.ssq_ld;
+  a.nrm_d = p.d;
+  a.eps = p.eps;
+  if (g.k == 0 || g.k == 2) a.ssq_in = p.ssq;   // input rows bf16(g * h): scaled by 1 / rms(h)
   if (g.dh_out) {
-    a.out_f32 = p.dh;
+    a.out_f32 = p.h;
     a.ldo = p.d;
+    // the next norm (of the gate/up or of the next layer's QKV) is folded into this epilogue; after
+    // the last layer the final norm normalises the selected rows from h
+    const __nv_bfloat16* gn = g.k == 1 ? p.mlp_norm[g.layer] : (g.layer + 1 < p.L ? p.attn_norm[g.layer + 1] : nullptr);
+    if (gn) {
+      a.gain = gn;
+      a.xg_out = p.x;
+      a.ssq_out = p.ssq;
+    }
   } else if (g.epi == EPI_F32) {
     a.out_f32 = p.logits;
     a.ldo = ITEM_ROWS_FWD;
@@ -295,64 +289,27 @@ __device__ GemmArgs epi_args(const FwdParams& p, const GP& g) {
   return a;
 }
 
-// Parts of the tiles of n-tile nt in the O / down projection gi: toff[mt] .. toff[mt + 1] index
-// tslot, the workspace slots of m-tile mt's parts in k order; a whole tile (one part) has none: its
-// product is in dh.  At most G + d / 128 entries.
-constexpr int PART_TABLE_CAP = 512;
-
+// Norm phases (256 compute threads).  final == false: layer 0's input rows -- the embedding rows
+// enter h, and x gets bf16(g * h) with the partial sums of squares (the norm's per-token scale is
+// applied by the QKV epilogue, as after every O / down projection).  final == true: RMSNorm of the
+// selected rows out_rows[r] of h into x row r, the LM head's input; the per-thread chunks and the
+// reduction are those of the 256-thread kernels, so the sums are the same bit for bit.  Between the
+// passes the row is kept in shared memory (`rowbuf`, d floats: the activation ring, idle then).
 template <int BN>
-__device__ void build_part_table(const FwdParams& p, int gi, int nt, int* toff, int* tslot, int ctid) {
-  const GP g = gemm_phase(p, gi, BN);
-  named_bar_sync(1, CT);   // earlier readers of the table are done
-  int cnt = 0, c_first = 0;
-  long long tu0 = 0;
-  if (ctid < g.m_tiles) {
-    const int t = ctid * g.n_tiles + nt;
-    if (t < g.w.r && g.to_dh) {   // a stream-K tile; whole (or GEMM-summed) tiles are in dh
-      tu0 = (long long)t * g.kb;
-      c_first = sk_owner(g.w, tu0);
-      cnt = sk_owner(g.w, tu0 + g.kb - 1) - c_first + 1;
-    }
-    if (cnt == 1) cnt = 0;
-    toff[ctid + 1] = cnt;
-  }
-  named_bar_sync(1, CT);
-  if (ctid == 0) {
-    toff[0] = 0;
-    for (int t = 1; t <= g.m_tiles; ++t) toff[t] += toff[t - 1];
-  }
-  named_bar_sync(1, CT);
-  if (ctid < g.m_tiles) {
-    for (int pi = 0; pi < cnt; ++pi) {
-      const int cc = c_first + pi;
-      const int e = toff[ctid] + pi;
-      if (e < PART_TABLE_CAP) tslot[e] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
-    }
-  }
-  if (ctid == 0 && toff[g.m_tiles] > PART_TABLE_CAP) set_error(p.err, ATSPEED_DEV_ERR_BOUNDS);
-  named_bar_sync(1, CT);
-}
-
-// RMSNorm of rows (256 compute threads; the per-thread chunks and the reduction are those of the
-// 256-thread kernels, so the sums are the same bit for bit).  mode 0 = embedding gather + norm
-// (layer 0); 1 = residual add h += (product of the preceding O / down projection gi_prev, summed
-// from its parts in k order starting from zero), then norm of h; 2 = the same for the selected rows
-// only (final norm).  Between the passes the row is kept in shared memory (`rowbuf`, d floats: the
-// activation ring, idle during a norm phase).
-constexpr int NORM_NB = 4;   // float4 chunks per thread in flight
-
-template <int BN>
-__device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const __nv_bfloat16* g, float* red,
-                                           float4* rowbuf, int ctid, int gi_prev, int* toff, int* tslot,
-                                           int& tab_nt, int ph) {
-  const int rows = mode == 2 ? p.n_out : p.T;
+__device__ __forceinline__ void norm_phase(const FwdParams& p, bool final, const __nv_bfloat16* g, float* red,
+                                           float4* rowbuf, int ctid, int ph) {
   const int d = p.d, nc = d / 4;
+  if (!final) {
+    for (int r = blockIdx.x; r < p.T; r += p.G)
+      embed_row(p.embed + (size_t)p.tok[r] * d, g, p.h + (size_t)r * d, p.x + (size_t)r * d, p.ssq, p.ssq_ld, r, d,
+                ctid, CT);
+    return;
+  }
   const int w = ctid >> 5, lane = ctid & 31;
-  for (int r = blockIdx.x; r < rows; r += p.G) {
-    const int src = mode == 2 ? p.out_rows[r] : r;
-    float* hr = p.h + (size_t)src * d;
+  for (int r = blockIdx.x; r < p.n_out; r += p.G) {
+    const float4* h4 = reinterpret_cast<const float4*>(p.h + (size_t)p.out_rows[r] * d);
     float ss = 0.f;
-    // the gains do not depend on the row: their loads go out with the first pass's
+    // the gains do not depend on the row: their loads go out with the row's
     constexpr int NG_MAX = 8192 / 4 / CT;   // chunks per thread, d <= 8192
     uint2 graw[NG_MAX];
 #pragma unroll
@@ -360,90 +317,12 @@ __device__ __forceinline__ void norm_phase(const FwdParams& p, int mode, const _
       const int c = ctid + CT * k;
       graw[k] = c < nc ? *reinterpret_cast<const uint2*>(g + 4 * c) : make_uint2(0, 0);
     }
-    if (mode == 0) {
-      const __nv_bfloat16* er = p.embed + (size_t)p.tok[r] * d;
-      for (int k0 = 0; k0 * CT < nc; k0 += NORM_NB) {
-        float4 v[NORM_NB];
 #pragma unroll
-        for (int k = 0; k < NORM_NB; ++k) {
-          const int c = ctid + CT * (k0 + k);
-          if (c < nc) {
-            const uint2 raw = *reinterpret_cast<const uint2*>(er + 4 * c);
-            const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&raw);
-            const float2 f0 = __bfloat1622float2(b[0]), f1 = __bfloat1622float2(b[1]);
-            v[k] = make_float4(f0.x, f0.y, f1.x, f1.y);
-          }
-        }
-#pragma unroll
-        for (int k = 0; k < NORM_NB; ++k) {
-          const int c = ctid + CT * (k0 + k);
-          if (c < nc) {
-            *reinterpret_cast<float4*>(hr + 4 * c) = v[k];
-            rowbuf[c] = v[k];
-            ss += v[k].x * v[k].x;
-            ss += v[k].y * v[k].y;
-            ss += v[k].z * v[k].z;
-            ss += v[k].w * v[k].w;
-          }
-        }
-      }
-    } else {
-      const int nt = src / BN, j = src - nt * BN;
-      if (gi_prev * 65536 + nt != tab_nt) {
-        build_part_table<BN>(p, gi_prev, nt, toff, tslot, ctid);
-        tab_nt = gi_prev * 65536 + nt;
-      }
-      // h += product: warp w takes m-tiles w, w + 8, ...; a lane four rows of each
-      const int mtn = (d + GEMM_BM - 1) / GEMM_BM;
-      const float4* ws4 = reinterpret_cast<const float4*>(p.ws);
-      constexpr long long SLOT4 = GEMM_WS_SLOT_FLOATS / 4;
-      const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int t0 = w; t0 < mtn; t0 += 32) {
-        float4 acc[4], hv[4];
-        int P[4], o[4];
-        int Pm = 0;
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-          const int mt = t0 + 8 * b;
-          const bool in = mt < mtn && mt * GEMM_BM + 4 * lane < d;
-          P[b] = in ? toff[mt + 1] - toff[mt] : 0;
-          o[b] = in ? toff[mt] : 0;
-          const size_t e = (size_t)src * d + mt * GEMM_BM + 4 * lane;
-          hv[b] = in ? __ldcg(reinterpret_cast<const float4*>(p.h + e)) : zero;
-          acc[b] = (in && P[b] == 0) ? __ldcg(reinterpret_cast<const float4*>(p.dh + e)) : zero;
-          Pm = max(Pm, P[b]);
-        }
-#pragma unroll 4
-        for (int e = 0; e < Pm; ++e) {
-          float4 v[4];
-#pragma unroll
-          for (int b = 0; b < 4; ++b)
-            if (e < P[b]) v[b] = __ldcg(ws4 + (long long)tslot[o[b] + e] * SLOT4 + j * (GEMM_BM / 4) + lane);
-#pragma unroll
-          for (int b = 0; b < 4; ++b) {
-            if (e < P[b]) {
-              acc[b].x += v[b].x;
-              acc[b].y += v[b].y;
-              acc[b].z += v[b].z;
-              acc[b].w += v[b].w;
-            }
-          }
-        }
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-          const int mt = t0 + 8 * b;
-          if (mt < mtn && mt * GEMM_BM + 4 * lane < d) {
-            const float4 v = make_float4(hv[b].x + acc[b].x, hv[b].y + acc[b].y, hv[b].z + acc[b].z,
-                                         hv[b].w + acc[b].w);
-            *reinterpret_cast<float4*>(hr + mt * GEMM_BM + 4 * lane) = v;   // the updated residual stream
-            rowbuf[mt * (GEMM_BM / 4) + lane] = v;
-          }
-        }
-      }
-      named_bar_sync(1, CT);
-      if (p.trace && ctid == 0 && r == (int)blockIdx.x) p.trace[((size_t)4 * (7 * p.L + 2) + ph) * p.G + blockIdx.x] = globaltimer_ns();
-      for (int c = ctid; c < nc; c += CT) {
-        const float4 v = rowbuf[c];
+    for (int k = 0; k < NG_MAX; ++k) {
+      const int c = ctid + CT * k;
+      if (c < nc) {
+        const float4 v = __ldcg(h4 + c);
+        rowbuf[c] = v;
         ss += v.x * v.x;
         ss += v.y * v.y;
         ss += v.z * v.z;
@@ -523,21 +402,20 @@ __device__ __forceinline__ bool attn_phase(const FwdParams& p, int l, uint8_t* a
 // a tile alternate between the two warpgroups (chunk ch by warpgroup ch & 1, each with its own
 // staging buffer and named barrier); warp 4 + q and warp 8 + q both read TMEM lane quadrant q.
 // For each of this CTA's segments, wait for its accumulator, then:
-//  * O / down projections (to_dh): a whole tile goes to dh, a split tile's part to this CTA's
-//    workspace slot ([token][row] layout); the next norm phase sums the parts;
-//  * other GEMMs: a whole tile runs the fused epilogue; for a split tile, if every other part is
-//    already published (and this is the CTA's last segment) this CTA is the last one and sums the
-//    parts with its own part read straight from TMEM; otherwise it publishes its part and the last
-//    CTA to arrive does the sum.
-//  * shared sums (phases with whole tiles per CTA, whose split tiles come first and finish early,
-//    and the LM head, whose tiles have many short parts): every part publishes, then each part sums
-//    a share of its tile's chunks (chunk ch by part ch mod parts).
-// Parts are always summed in k order starting from zero, whichever CTA sums them.  Kept out of
-// line so that the epilogue gets its own register allocation.
+//  * a whole tile runs the fused epilogue; for a split tile, if every other part is already
+//    published (and this is the CTA's last segment) this CTA is the last one and sums the parts
+//    with its own part read straight from TMEM; otherwise it publishes its part and the last CTA
+//    to arrive does the sum;
+//  * shared sums (phases with whole tiles per CTA, whose split tiles come first and finish early;
+//    the O / down projections, whose residual update ends the phase; the LM head, whose tiles have
+//    many short parts): every part publishes, then each part sums a share of its tile's chunks
+//    (chunk ch by part ch mod parts).
+// Parts are always summed in k order starting from zero, whichever CTA sums them.  The QKV and
+// gate/up epilogues first multiply by each token's norm scale (trs, loaded per token tile).
 template <int BN>
 __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int ph, float* staging_base, uint64_t* tfull,
-                                            uint64_t* tempty, int* flag, int* part_slot, int* tpos, int* tkvr,
-                                            GemmArgs* s_ea, uint32_t tmem_base, int ctid, int& si) {
+                                               uint64_t* tempty, int* flag, int* part_slot, int* tpos, int* tkvr,
+                                               float* trs, GemmArgs* s_ea, uint32_t tmem_base, int ctid, int& si) {
   const int c = blockIdx.x, G = p.G, NP = 7 * p.L + 2;
   const int wg = ctid >> 7, wt = ctid & 127, wbar = 2 + wg;
   // a warp reads the TMEM lane quadrant of its warp id mod 4; each warpgroup (4 consecutive warps)
@@ -550,6 +428,18 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
   named_bar_sync(1, CT);
   const GemmArgs& ea = *s_ea;
   const int kb = g.kb;
+  const bool scaled = g.k == 0 || g.k == 2;
+  const float* trs_e = scaled ? trs : nullptr;
+  // per-token tables of the token tile nt (QKV: rotary positions and cache rows; QKV and gate/up:
+  // norm scales), loaded when the tile changes; callers synchronise before their first use
+  int tab_nt = -1;
+  auto tables = [&](int nt) {
+    if ((g.epi != EPI_QKV && !scaled) || nt == tab_nt) return;
+    named_bar_sync(1, CT);   // both warpgroups are done with the previous tables
+    tab_nt = nt;
+    if (g.epi == EPI_QKV) load_tok_tables<BN>(ea, nt, tpos, tkvr, ctid, CT);
+    if (scaled) load_norm_scales<BN>(ea, nt, trs, ctid, CT);
+  };
   SegIter it;
   it.init(g.w, c);
   int tile, k0, k1;
@@ -559,17 +449,7 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
       part_slot[pi] = cc * 2 + (sk_start(g.w, cc) >= tu0 ? 0 : 1);
     }
   };
-  // a bulk copy of a split part (O / down projections) must have finished, in global memory and
-  // before its staging buffer is reused, when the phase ends (the next phases read the part with
-  // generic loads after the grid barrier, hence the proxy fence)
-  auto drain = [&]() {
-    if (wt == 0) {
-      bulk_wait_done();
-      fence_proxy_async();
-    }
-  };
-  const bool shared_sums =
-      !g.to_dh && (g.w.q > 0 || g.dh_out || (gi == 4 * p.L && g.w.Gsk > 0 && g.w.Usk / g.w.Gsk + 1 < kb));
+  const bool shared_sums = g.w.q > 0 || g.dh_out || (gi == 4 * p.L && g.w.Gsk > 0 && g.w.Usk / g.w.Gsk + 1 < kb);
   if (shared_sums && it.u < it.u1) {
     int sk_tile[2], nsk = 0;
     while (it.u < it.u1 && nsk < 2) {
@@ -577,7 +457,7 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
       const int acc = si & 1, use = si >> 1;
       ++si;
       const bool got = named_bar_and(1, CT, mwait(&tfull[acc], (uint32_t)(use & 1), p.err));
-      if (!got) { drain(); return false; }
+      if (!got) return false;
       tc_fence_after();
       const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       const int nch = min(BN / 32, (g.rows - (tile % g.n_tiles) * BN + 31) / 32);
@@ -598,17 +478,17 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
       const int parts = sk_owner(g.w, tu0 + kb - 1) - c_first + 1;
       const int m_tile = t / g.n_tiles, n_tile = t % g.n_tiles;
       fill_part_slots(tu0, c_first, parts);
-      if (g.epi == EPI_QKV) load_tok_tables<BN>(ea, n_tile, tpos, tkvr, ctid, CT);
+      tables(n_tile);
       if (ctid == 0) *flag = counter_wait(&skc[t], parts, p.err) ? 1 : 0;
       named_bar_sync(1, CT);
-      if (!*flag) { drain(); return false; }
+      if (!*flag) return false;
       const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
       int k = 0;
       for (int ch = c - c_first; ch < nch; ch += parts, ++k) {
         if ((k & 1) != wg) continue;
         ws_reduce_chunk<1>(p.ws, part_slot, parts, ch, m, staging);
         named_bar_sync(wbar, 128);
-        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr, trs_e, wbar);
         named_bar_sync(wbar, 128);
       }
       named_bar_sync(1, CT);   // flag, part_slot and the token tables are reused
@@ -618,13 +498,10 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
     const int acc = si & 1, use = si >> 1;
     const int m_tile = tile / g.n_tiles, n_tile = tile % g.n_tiles;
     const bool whole = (k0 == 0 && k1 == kb);
-    if (g.epi == EPI_QKV) {
-      named_bar_sync(1, CT);   // both warpgroups are done with the previous segment's token tables
-      load_tok_tables<BN>(ea, n_tile, tpos, tkvr, ctid, CT);
-    }
+    tables(n_tile);
     long long tu0 = 0;
     int c_first = 0, parts = 1;
-    if (!whole && !g.to_dh) {
+    if (!whole) {
       tu0 = (long long)tile * kb;
       c_first = sk_owner(g.w, tu0);
       parts = sk_owner(g.w, tu0 + kb - 1) - c_first + 1;
@@ -632,59 +509,11 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
     }
     // (the vote is also the barrier after which token tables and part slots are in place)
     const bool got = named_bar_and(1, CT, mwait(&tfull[acc], (uint32_t)(use & 1), p.err));
-    if (!got) { drain(); return false; }
+    if (!got) return false;
     tc_fence_after();
     if (p.trace && ctid == 0) p.trace[((size_t)4 * NP + ph) * G + c] = globaltimer_ns();
     const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
     const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
-    const int row = m_tile * GEMM_BM + m;
-    if (g.to_dh && !whole) {
-      // split part, [token][128 rows] fp32 in this CTA's workspace slot, where a 32-token chunk is
-      // 16 KB in one piece: TMEM -> the warpgroup's staging buffer -> one bulk copy per chunk
-      // (issued by one thread; the staging buffer is reused once that copy has read it)
-      float* slot = p.ws + ((long long)c * 2 + (seg == 0 ? 0 : 1)) * GEMM_WS_SLOT_FLOATS;
-      for (int ch = wg; ch < nch; ch += 2) {
-        uint32_t r[32];
-        tmem_ld_32x32b_x32(tb + ch * 32, r);
-        tmem_ld_wait();
-        const int nv = min(32, g.rows - n_tile * BN - ch * 32);
-        if (wt == 0) bulk_wait_read();
-        named_bar_sync(wbar, 128);
-#pragma unroll
-        for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = __uint_as_float(r[j]);
-        fence_proxy_async_smem();   // the generic stores before the bulk copy's async reads
-        named_bar_sync(wbar, 128);
-        if (wt == 0) bulk_store(slot + (size_t)ch * 32 * GEMM_BM, staging, (uint32_t)nv * GEMM_BM * 4);
-      }
-      tc_fence_before();
-      if (lane == 0) mbar_arrive(&tempty[acc]);
-      continue;
-    }
-    if (g.to_dh) {
-      float* dst;
-      size_t ld;
-      if (whole) {
-        dst = p.dh + (size_t)n_tile * BN * p.d + row;
-        ld = (size_t)p.d;
-      } else {
-        dst = p.ws + ((long long)c * 2 + (seg == 0 ? 0 : 1)) * GEMM_WS_SLOT_FLOATS + m;
-        ld = GEMM_BM;
-      }
-      for (int ch = wg; ch < nch; ch += 2) {
-        uint32_t r[32];
-        tmem_ld_32x32b_x32(tb + ch * 32, r);
-        tmem_ld_wait();
-        const int nv = min(32, g.rows - n_tile * BN - ch * 32);
-        if (!whole || row < g.M) {
-#pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (j < nv) __stcg(dst + (size_t)(ch * 32 + j) * ld, __uint_as_float(r[j]));
-        }
-      }
-      tc_fence_before();
-      if (lane == 0) mbar_arrive(&tempty[acc]);
-      continue;
-    }
     if (whole) {
       for (int ch = wg; ch < nch; ch += 2) {
         uint32_t r[32];
@@ -693,7 +522,7 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
 #pragma unroll
         for (int j = 0; j < 32; ++j) staging[j * GEMM_BM + m] = __uint_as_float(r[j]);
         named_bar_sync(wbar, 128);
-        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr, trs_e, wbar);
         named_bar_sync(wbar, 128);
       }
       tc_fence_before();
@@ -717,7 +546,7 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
         tmem_ld_wait();
         ws_reduce_chunk_own(p.ws, part_slot, parts, own, r, ch, m, staging);
         named_bar_sync(wbar, 128);
-        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr, trs_e, wbar);
         named_bar_sync(wbar, 128);
       }
       tc_fence_before();
@@ -747,13 +576,12 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
       for (int ch = wg; ch < nch; ch += 2) {
         ws_reduce_chunk<1>(p.ws, part_slot, parts, ch, m, staging);
         named_bar_sync(wbar, 128);
-        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr);
+        epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr, trs_e, wbar);
         named_bar_sync(wbar, 128);
       }
     }
     named_bar_sync(1, CT);  // flag and part_slot are reused by the next segment
   }
-  drain();
   return true;
 }
 
@@ -787,11 +615,10 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
   int* part_slot = reinterpret_cast<int*>(red + 8);               // 256
   int* tpos = part_slot + 256;                                    // [BN] QKV token tables
   int* tkvr = tpos + 256;
-  int* toff = tkvr + 256;                                         // [65] part table (norm phases)
-  int* tslot = toff + 68;                                         // [PART_TABLE_CAP]
-  GemmArgs* s_ea = reinterpret_cast<GemmArgs*>((reinterpret_cast<uintptr_t>(tslot + PART_TABLE_CAP) + 15) &
+  float* trs = reinterpret_cast<float*>(tkvr + 256);              // [BN] norm scales (QKV, gate/up)
+  GemmArgs* s_ea = reinterpret_cast<GemmArgs*>((reinterpret_cast<uintptr_t>(trs + 256) + 15) &
                                                 ~uintptr_t(15));   // epilogue arguments
-  static_assert(8 * (2 * C::SA + 2 * C::SB + 9) + 4 * (6 + C::SA + C::SB + 8 + 256 + 512 + 68 + PART_TABLE_CAP) + 16 + (int)sizeof(GemmArgs) <=
+  static_assert(8 * (2 * C::SA + 2 * C::SB + 9) + 4 * (6 + C::SA + C::SB + 8 + 256 + 768) + 16 + (int)sizeof(GemmArgs) <=
                     C::MISC,
                 "shared-memory misc area too small");
 
@@ -970,8 +797,8 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
     const int wg = ctid >> 7, wt = ctid & 127;
     int si = 0;
     int use_att[2] = {0, 0};
-    int tab_nt = -1;   // (GEMM phase, n-tile) whose part table is in toff / tslot
     bool ok = true;
+    int nb = 0;   // grid barriers passed
     for (int ph = 0; ph < NP && ok; ++ph) {
       // which phase is this?
       int kind, l = 0;   // 0 NORM0, 1 GEMM, 2 ATTN, 3 NORM (mlp), 4 NORM (next attn / final)
@@ -995,27 +822,18 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
           kind = 4;
         }
       }
-      if ((kind == 3 || kind == 4) && ph > 0) {
-        // the part table of this CTA's first row does not depend on data: build it before the wait
-        const int r0 = blockIdx.x;
-        const bool fin = kind == 4 && l + 1 == L;
-        if (r0 < (fin ? p.n_out : p.T)) {
-          const int nt = (fin ? p.out_rows[r0] : r0) / BN;
-          const int gp = 4 * l + (kind == 3 ? 1 : 3);
-          if (gp * 65536 + nt != tab_nt) {
-            build_part_table<BN>(p, gp, nt, toff, tslot, ctid);
-            tab_nt = gp * 65536 + nt;
-          }
-        }
-      }
+      // the norms before the gate/up projection and before the next layer's QKV are folded into
+      // the GEMMs around them: no phase, no barrier
+      if (kind == 3 || (kind == 4 && l + 1 < L)) continue;
       if (ph > 0) {
-        // Barrier ph-1 must be complete before this CTA can arrive at barrier ph: the arrival counter
+        // Barrier nb-1 must be complete before this CTA can arrive at barrier nb: the arrival counter
         // is shared by all barriers, so an early arrival would count towards the previous one.
         // (Non-GEMM phases also read what the previous phase wrote.)
         if (ctid == 0) {
-          *flag = grid_wait(p, ph - 1) ? 1 : 0;
+          *flag = grid_wait(p, nb) ? 1 : 0;
           if (*flag && kind == 1) st_release_cta(go, gi + 1);
         }
+        ++nb;
         named_bar_sync(1, CT);
         if (!*flag) {
           ok = false;
@@ -1024,11 +842,8 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
         fence_proxy_async();
         named_bar_sync(1, CT);
       }
-      if (kind == 0 || kind == 3 || kind == 4) {
-        const int nmode = kind == 0 ? 0 : (kind == 4 && l + 1 == L) ? 2 : 1;
-        const __nv_bfloat16* ng = kind == 0 ? p.attn_norm[0] : kind == 3 ? p.mlp_norm[l]
-                                  : (l + 1 < L ? p.attn_norm[l + 1] : p.final_norm);
-        norm_phase<BN>(p, nmode, ng, red, rowbuf, ctid, 4 * l + (kind == 3 ? 1 : 3), toff, tslot, tab_nt, ph);
+      if (kind == 0 || kind == 4) {
+        norm_phase<BN>(p, kind == 4, kind == 0 ? p.attn_norm[0] : p.final_norm, red, rowbuf, ctid, ph);
       } else if (kind == 2) {
         // both warpgroups leave together: a failed bounded wait in either ends the program
         const bool aok = attn_phase<HD>(p, l, att_smem + wg * LY::ATT_BODY, att_bars + 2 * wg,
@@ -1038,7 +853,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
           break;
         }
       } else {
-        if (!gemm_epi_phase<BN>(p, gi, ph, staging, tfull, tempty, flag, part_slot, tpos, tkvr, s_ea, tmem_base, ctid, si)) {
+        if (!gemm_epi_phase<BN>(p, gi, ph, staging, tfull, tempty, flag, part_slot, tpos, tkvr, trs, s_ea, tmem_base, ctid, si)) {
           ok = false;
           break;
         }

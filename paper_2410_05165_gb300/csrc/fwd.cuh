@@ -1,6 +1,6 @@
 // Persistent forward kernel: one cooperative launch runs a whole decoder forward (every layer's
-// RMSNorm, QKV GEMM + RoPE + KV store, tree attention, O GEMM + residual, RMSNorm, gate/up GEMM +
-// SwiGLU, down GEMM + residual, then the final norm and the item-code LM head).
+// QKV GEMM + RMSNorm scale + RoPE + KV store, tree attention, O GEMM + residual, gate/up GEMM +
+// RMSNorm scale + SwiGLU, down GEMM + residual, then the final norm and the item-code LM head).
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -34,8 +34,11 @@ struct FwdParams {
   const __nv_bfloat16* embed;
   // activations
   float* h;                 // [T][d] fp32 residual stream
-  float* dh;                // [T][d] fp32 product of the last O / down projection, added to h by the norm
-  __nv_bfloat16* x;         // [Xrows][d] normalised rows (GEMM B operand)
+  float* ssq;               // [ceil(d / 128)][ssq_ld] partial sums of squares of h per 128-row tile
+  int ssq_ld;
+  __nv_bfloat16* x;         // [Xrows][d] B operand of the QKV / gate-up GEMMs: bf16(g * h) (the norm's
+                            // per-token scale is applied in their epilogues); the LM head's: the
+                            // final norm's rows
   __nv_bfloat16* q;         // [T][d]
   __nv_bfloat16* att;       // [Xrows][d]
   __nv_bfloat16* act;       // [Xrows][ffn]

@@ -1,6 +1,6 @@
 // Weight-streaming GEMM for sm_103a: TMA -> shared memory (128B swizzle) -> tcgen05.mma with the
 // fp32 accumulator in TMEM -> tcgen05.ld epilogue with fused QKV+RoPE+KV-store / SwiGLU /
-// residual-add / plain stores.
+// residual-add (with the next RMSNorm's partial sums) / plain stores.
 //
 // Decomposition ("stream-K"): the work units are (tile, 64-wide k-block) pairs, tile = (weight-row
 // tile of 128, token tile of BN), ordered weight-tile-major.  A persistent grid of one CTA per SM
@@ -38,7 +38,8 @@ struct Cfg {
   static constexpr int B_BYTES = BN * 128;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGING_FLOATS = 32 * BM;
-  static constexpr int BAR_BYTES = 256 + 1024 + 2048;  // barriers, flags, split-part slot table, token tables
+  static constexpr int BAR_BYTES = 256 + 1024 + 2048 + 1024;  // barriers, flags, split-part slot table, token
+                                                              // tables, norm scales
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_FLOATS * 4 + BAR_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
 };
@@ -75,6 +76,7 @@ __global__ void __launch_bounds__(192, 1)
   int* part_slot = last_fill + 8;  // [<= 256] workspace slots of a split tile's parts
   int* tpos = part_slot + 256;     // [BN] QKV epilogue token tables of the current n-tile
   int* tkvr = tpos + 256;
+  float* trs = reinterpret_cast<float*>(tkvr + 256);   // [BN] norm scales of the current n-tile
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x;
@@ -235,6 +237,14 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const int m_tile = tile / p.n_tiles, n_tile = tile % p.n_tiles;
       if constexpr (EPI == EPI_QKV) load_tok_tables<BN>(p.a, n_tile, tpos, tkvr, ep_tid);
+      const bool scaled = (EPI == EPI_QKV || EPI == EPI_SWIGLU) && p.a.ssq_in != nullptr;
+      if (scaled) load_norm_scales<BN>(p.a, n_tile, trs, ep_tid, 128);
+      auto epilogue = [&](int ch) {
+        if constexpr (EPI == EPI_RESNORM)
+          epi_resnorm(p.a, staging, m_tile, n_tile * BN + ch * 32, ep_tid, 1);
+        else
+          epi_chunk<BN, EPI>(p.a, staging, m_tile, n_tile, ch, ep_tid, tpos, tkvr, scaled ? trs : nullptr);
+      };
       const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       // 32-token chunks that hold at least one valid token (the rest are padding)
       const int nch = min(BN / 32, (p.a.T - n_tile * BN + 31) / 32);
@@ -246,7 +256,7 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
           for (int j = 0; j < 32; ++j) staging[j * BM + m] = __uint_as_float(r[j]);
           named_bar_sync(1, 128);
-          epi_chunk<BN, EPI>(p.a, staging, m_tile, n_tile, ch, ep_tid, tpos, tkvr);
+          epilogue(ch);
           named_bar_sync(1, 128);
         }
         tc_fence_before();
@@ -281,7 +291,7 @@ __global__ void __launch_bounds__(192, 1)
           for (int ch = 0; ch < nch; ++ch) {
             ws_reduce_chunk(p.ws, part_slot, parts, ch, m, staging);
             named_bar_sync(1, 128);
-            epi_chunk<BN, EPI>(p.a, staging, m_tile, n_tile, ch, ep_tid, tpos, tkvr);
+            epilogue(ch);
             named_bar_sync(1, 128);
           }
         }
@@ -366,6 +376,7 @@ cudaError_t launch_bn(EpiKind e, const CUtensorMap& ma, const CUtensorMap& mb, c
     case EPI_SWIGLU: return launch_t<BN, EPI_SWIGLU>(ma, mb, kp, st, pdl);
     case EPI_QKV: return launch_t<BN, EPI_QKV>(ma, mb, kp, st, pdl);
     case EPI_LSE: return launch_t<BN, EPI_LSE>(ma, mb, kp, st, pdl);
+    case EPI_RESNORM: return launch_t<BN, EPI_RESNORM>(ma, mb, kp, st, pdl);
   }
   return cudaErrorInvalidValue;
 }

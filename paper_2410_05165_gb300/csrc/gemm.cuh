@@ -8,7 +8,7 @@
 
 namespace atspeed {
 
-enum EpiKind : int { EPI_F32 = 0, EPI_BF16 = 1, EPI_RESID = 2, EPI_SWIGLU = 3, EPI_QKV = 4, EPI_LSE = 5 };
+enum EpiKind : int { EPI_F32 = 0, EPI_BF16 = 1, EPI_RESID = 2, EPI_SWIGLU = 3, EPI_QKV = 4, EPI_LSE = 5, EPI_RESNORM = 6 };
 
 // Y[t][m] = sum_k W[m][k] * X[t][k]  (W: weight rows, X: token rows, both bf16 K-major)
 // with a fused epilogue.  The MMA runs "swap-AB": weight rows are the MMA M dimension (128 per
@@ -22,8 +22,21 @@ struct GemmArgs {
   int K;                    // reduction length, multiple of 64
   int T;                    // tokens
   int X_rows;               // allocated token rows of X
+  // RMSNorm folded into the GEMMs around it (LLaMA pre-norm: x = h / rms(h) * g; the per-token
+  // scale 1 / rms(h) commutes with the projection, so W x = (W (g h)) / rms(h)):
+  //  * EPI_RESNORM (O / down projections): h += product, then xg = bf16(g * h) and, per 128-row
+  //    tile mt of h, the token's partial sum of squares ssq[mt * ssq_ld + t];
+  //  * EPI_QKV / EPI_SWIGLU with ssq_in set: the product is multiplied by the token's
+  //    1 / sqrt(sum_mt ssq[mt][t] / nrm_d + eps) before the epilogue's arithmetic.
+  const float* ssq_in;      // partial sums of the GEMM input's rows (null: no scaling)
+  float* ssq_out;           // EPI_RESNORM: partial sums of the updated residual (null: none)
+  int ssq_ld;               // token stride of the partial sums
+  int nrm_d;                // norm width (d_model); its ceil(d / 128) tiles are summed
+  float eps;
+  const __nv_bfloat16* gain;  // EPI_RESNORM: gain of the next norm (null: only h is written)
+  __nv_bfloat16* xg_out;      // EPI_RESNORM: [T][ldo] bf16(g * h), the next GEMM's input
   // outputs
-  float* out_f32;           // EPI_F32 / EPI_RESID: [T][ldo]
+  float* out_f32;           // EPI_F32 / EPI_RESID / EPI_RESNORM: [T][ldo]
   __nv_bfloat16* out_bf16;  // EPI_BF16 / EPI_SWIGLU: [T][ldo]
   int ldo;
   // EPI_LSE: per (weight-row tile, token) the tile's (max, sum of exp(y - max)) over its rows,

@@ -131,11 +131,86 @@ __device__ __forceinline__ void load_tok_tables(const GemmArgs& a, int n_tile, i
   }
 }
 
+// ---- RMSNorm folded into the GEMMs around it
+// Sum of squares of 32 values v(0 .. 31) in the rotated order rot, rot + 1, ... (mod 32), one fused
+// multiply-add per value.  A token's partial sum over a 128-row tile of the residual is
+// (q0 + q1) + (q2 + q3), q_s = ssq32 over rows 32 s .. 32 s + 31 of the tile with rot =
+// ssq_rot(s, token); rows past d count as zero.  Every producer of partial sums (the O / down
+// epilogue, the embedding rows) uses exactly these orders, so a token's sums do not depend on the
+// kernel or the schedule that made them.
+template <class F>
+__device__ __forceinline__ float ssq32(F v, int rot) {
+  float s = 0.f;
+#pragma unroll 8
+  for (int i = 0; i < 32; ++i) {
+    const float x = v((i + rot) & 31);
+    s = __fmaf_rn(x, x, s);
+  }
+  return s;
+}
+__device__ __forceinline__ int ssq_rot(int sub, int tok) { return (sub * 8 + (tok & 31)) & 31; }
+
+// 1 / rms of token t (RMSNorm's per-token scale) from its partial sums, added in tile order.
+__device__ __forceinline__ float norm_scale(const float* ssq, int ld, int d, float eps, int t) {
+  const int nt = (d + GEMM_BM - 1) / GEMM_BM;
+  float s = 0.f;
+#pragma unroll 8
+  for (int mt = 0; mt < nt; ++mt) s += __ldcg(ssq + (size_t)mt * ld + t);
+  return 1.0f / sqrtf(s / (float)d + eps);
+}
+
+// The scales of the BN tokens of n-tile n_tile into trs (shared memory); callers synchronise
+// before the epilogue reads them.
+template <int BN>
+__device__ __forceinline__ void load_norm_scales(const GemmArgs& a, int n_tile, float* trs, int tid, int nthreads) {
+  for (int j = tid; j < BN; j += nthreads) {
+    const int tok = n_tile * BN + j;
+    trs[j] = tok < a.T ? norm_scale(a.ssq_in, a.ssq_ld, a.nrm_d, a.eps, tok) : 0.f;
+  }
+}
+
+// EPI_RESNORM over one 32-token chunk (O / down projections): h += product (fp32 residual,
+// read-modify-write; every (row, token) belongs to one chunk of one CTA), xg = bf16(g * h) for the
+// next GEMM, and the partial sums of squares of the updated rows.  128 threads (ep_tid = the tile
+// row they own); `bar` is a named barrier of those 128 threads.  st (staging, [32 tokens][128 rows])
+// holds the product and is overwritten with the updated residual.
+__device__ __forceinline__ void epi_resnorm(const GemmArgs& a, float* st, int m_tile, int tok0, int ep_tid, int bar) {
+  const int nv = min(32, a.T - tok0);
+  const int m = ep_tid, row = m_tile * GEMM_BM + m;
+  const bool in = row < a.M;
+  float* base = a.out_f32 + (size_t)tok0 * a.ldo + row;
+  const bool xg = a.gain != nullptr;
+  const float g = (in && xg) ? __bfloat162float(a.gain[row]) : 0.f;
+  float old[32];
+#pragma unroll
+  for (int n = 0; n < 32; ++n) old[n] = (in && n < nv) ? __ldcg(base + (size_t)n * a.ldo) : 0.f;
+#pragma unroll
+  for (int n = 0; n < 32; ++n) {
+    const float v = in ? old[n] + st[n * GEMM_BM + m] : 0.f;
+    if (in && n < nv) {
+      base[(size_t)n * a.ldo] = v;
+      if (xg) a.xg_out[(size_t)(tok0 + n) * a.ldo + row] = __float2bfloat16_rn(v * g);
+    }
+    st[n * GEMM_BM + m] = v;
+  }
+  if (a.ssq_out == nullptr) return;
+  named_bar_sync(bar, 128);
+  // token j of the chunk (j = its index mod 32), quarter sub of the rows; the rotation also spreads
+  // a warp's shared-memory reads over the 32 banks
+  const int j = ep_tid >> 2, sub = ep_tid & 3;
+  const float* sj = st + j * GEMM_BM + sub * 32;
+  float s = ssq32([&](int r) { return sj[r]; }, ssq_rot(sub, j));
+  s += __shfl_xor_sync(0xffffffffu, s, 1);
+  s += __shfl_xor_sync(0xffffffffu, s, 2);
+  if (sub == 0 && j < nv) a.ssq_out[(size_t)m_tile * a.ssq_ld + tok0 + j] = s;
+}
+
 // st: staging [32 tokens][128 rows] fp32 of one chunk; 128 threads (ep_tid) write the outputs.
-// tpos / tkvr: the n-tile's token tables (EPI_QKV only).
+// tpos / tkvr: the n-tile's token tables (EPI_QKV only); trs: the n-tile's norm scales (EPI_QKV /
+// EPI_SWIGLU when the input rows are g * h, else null).
 template <int BN, int EPI>
 __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, int m_tile, int n_tile, int ch,
-                                          int ep_tid, const int* tpos, const int* tkvr) {
+                                          int ep_tid, const int* tpos, const int* tkvr, const float* trs = nullptr) {
   const int tok0 = n_tile * BN + ch * 32;
   if constexpr (EPI == EPI_QKV) {
     // rows of q | k | v.  Thread = (two adjacent rotation pairs, token quarter): pairs (i, i + hd/2)
@@ -159,8 +234,15 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, in
         const int n = n0 + 4 * k;
         if (n < nv) {
           __half* vr = a.v_cache + (size_t)tkvr[tt0 + n] * d;
-          const float2 lo = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_lo);
-          const float2 hi = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_hi);
+          float2 lo = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_lo);
+          float2 hi = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_hi);
+          if (trs) {
+            const float sc = trs[tt0 + n];
+            lo.x *= sc;
+            lo.y *= sc;
+            hi.x *= sc;
+            hi.y *= sc;
+          }
           *reinterpret_cast<__half2*>(vr + f_lo) =
               __halves2half2(__float2half_rn(bf16_round(lo.x)), __float2half_rn(bf16_round(lo.y)));
           *reinterpret_cast<__half2*>(vr + f_hi) =
@@ -180,8 +262,15 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, in
       for (int k = 0; k < 8; ++k) {
         const int n = n0 + 4 * k;
         if (n < nv) {
-          const float2 xl = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_lo);
-          const float2 xh = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_hi);
+          float2 xl = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_lo);
+          float2 xh = *reinterpret_cast<const float2*>(st + n * GEMM_BM + r_hi);
+          if (trs) {
+            const float sc = trs[tt0 + n];
+            xl.x *= sc;
+            xl.y *= sc;
+            xh.x *= sc;
+            xh.y *= sc;
+          }
           const __nv_bfloat16 o_lo0 = __float2bfloat16_rn(xl.x * cth[k].x - xh.x * sth[k].x);
           const __nv_bfloat16 o_hi0 = __float2bfloat16_rn(xh.x * cth[k].x + xl.x * sth[k].x);
           const __nv_bfloat16 o_lo1 = __float2bfloat16_rn(xl.y * cth[k].y - xh.y * sth[k].y);
@@ -208,6 +297,13 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const float* st, in
       const int n = n0 + 4 * k;
       gv[k] = *reinterpret_cast<const float2*>(st + n * GEMM_BM + 2 * f);
       uv[k] = *reinterpret_cast<const float2*>(st + n * GEMM_BM + 64 + 2 * f);
+      if (trs) {
+        const float sc = trs[ch * 32 + n];
+        gv[k].x *= sc;
+        gv[k].y *= sc;
+        uv[k].x *= sc;
+        uv[k].y *= sc;
+      }
     }
 #pragma unroll
     for (int k = 0; k < 8; ++k) {

@@ -13,6 +13,11 @@ cudaError_t rmsnorm_launch(const float* h, const int* tokens, const __nv_bfloat1
                            const __nv_bfloat16* g, int T, int d, float eps, __nv_bfloat16* x, int ldx,
                            cudaStream_t st, bool pdl);
 
+// Layer 0's rows with the first norm folded into the QKV GEMM: h[t] = embed[tokens[t]],
+// xg[t] = bf16(g * h[t]), ssq[mt * ld + t] = partial sums of squares of h[t] per 128-row tile.
+cudaError_t embed_rows_launch(const int* tokens, const __nv_bfloat16* embed, const __nv_bfloat16* g, float* h,
+                              __nv_bfloat16* xg, float* ssq, int ld, int T, int d, cudaStream_t st, bool pdl);
+
 // x[i] = bf16(rmsnorm(h[rows[i]]) * g) for i < n (final norm of the tokens whose logits are needed)
 cudaError_t rmsnorm_rows_launch(const float* h, const int* rows, int n, const __nv_bfloat16* g, int d, float eps,
                                 __nv_bfloat16* x, int ldx, cudaStream_t st, bool pdl);

@@ -7,7 +7,8 @@ that comes out the other way (fp32 tensor-core sums against the oracle's fp64) p
 all later layers.  Here every layer of the oracle runs on the GPU's OWN input to that layer, and
 each rounding point of the layer is compared on its own:
 
-* q, k, v after RoPE (bf16), from the GPU's residual entering the layer;
+* q, k, v after RoPE (bf16), from the GPU's residual entering the layer (the GEMM input is the
+  gain-scaled residual g * h in bf16, the norm's per-token scale multiplies the GEMM output);
 * the tree attention output (bf16), from the GPU's q and its K/V cache (history pages written by
   the prefill, path keys written by this forward);
 * the SwiGLU product (bf16), from the GPU's attention output (O projection, residual and RMSNorm in
@@ -33,7 +34,7 @@ import torch
 import synth
 from oracle.model import (Model, _attend, _layer_mlp_act, _layer_mlp_out, _layer_pre_attn,
                           final_hidden_to_logits)
-from oracle.numerics import bf16, rmsnorm, rope_angles, silu
+from oracle.numerics import bf16, rms_scale, rmsnorm, rope_angles, silu
 
 pytestmark = pytest.mark.gpu
 
@@ -151,12 +152,17 @@ def _run_case(ats, cfg, n_layers, prompts, K, N, G, items_n, seed_tree=5):
         pos = g.pos.astype(np.int64)
         # ---- q, k, v from the GPU's residual
         q_ref, k_ref, v_ref = _layer_pre_attn(m, l, h_in, pos)
-        x = bf16(rmsnorm(h_in, m.W(f"layers.{l}.attn_norm"), spec.rms_eps))
+        # GEMM input g * h (bf16; the fp32 product rounds first), output times the norm scale
+        # s(h), which the GPU sums in fp32 from per-tile partial sums (relative error < 2^-18)
+        xgr = h_in * m.W(f"layers.{l}.attn_norm")
+        xg = bf16(xgr)
+        rs = rms_scale(h_in, spec.rms_eps)
         W = np.asarray(tw[f"layers.{l}.wqkv"], np.float32)
         Wa = np.abs(W)
-        xr = rmsnorm(h_in, m.W(f"layers.{l}.attn_norm"), spec.rms_eps)
-        slack = 4 * U32 * np.sqrt(d) * (np.abs(x).astype(np.float32) @ Wa.T).astype(np.float64)
-        slack += (_flip_risk(xr, 2.0 ** -20) * _ulp(xr)).astype(np.float32) @ Wa.T
+        mag = (np.abs(xg).astype(np.float32) @ Wa.T).astype(np.float64)
+        slack = 4 * U32 * np.sqrt(d) * mag
+        slack += (_flip_risk(xgr, 2.0 ** -23) * _ulp(xgr)).astype(np.float32) @ Wa.T
+        slack = slack * rs + 2.0 ** -18 * mag * rs
         ang = rope_angles(pos, hd, spec.rope_theta)
         cs, sn = np.abs(np.cos(ang))[:, None, :], np.abs(np.sin(ang))[:, None, :]
 
@@ -194,14 +200,18 @@ def _run_case(ats, cfg, n_layers, prompts, K, N, G, items_n, seed_tree=5):
         Wo = np.abs(np.asarray(tw[f"layers.{l}.wo"], np.float32))
         dh_mid = 4 * U32 * np.sqrt(d) * (np.abs(g.att).astype(np.float32) @ Wo.T).astype(np.float64)
         gn = m.W(f"layers.{l}.mlp_norm")
-        x2r = rmsnorm(h_mid, gn, spec.rms_eps)
-        rs = 1.0 / np.sqrt(np.mean(h_mid * h_mid, axis=-1, keepdims=True) + spec.rms_eps)
-        rel = (dh_mid * rs * np.abs(gn)) / np.maximum(np.abs(x2r), 1e-30) + 2.0 ** -20
+        x2r = h_mid * gn
+        rs = rms_scale(h_mid, spec.rms_eps)
+        # the GPU's residual carries the O projection's fp32 error dh_mid: into g * h, and into s(h)
+        rel = (dh_mid * np.abs(gn)) / np.maximum(np.abs(x2r), 1e-30) + 2.0 ** -20
+        rel_rs = np.sum(np.abs(h_mid) * dh_mid, axis=-1, keepdims=True) / np.sum(h_mid * h_mid, axis=-1, keepdims=True)
         x2 = bf16(x2r)
         Wgu = np.abs(np.asarray(tw[f"layers.{l}.wgate_up"], np.float32))
-        acc = 4 * U32 * np.sqrt(d) * (np.abs(x2).astype(np.float32) @ Wgu.T).astype(np.float64)
+        mag = (np.abs(x2).astype(np.float32) @ Wgu.T).astype(np.float64)
+        acc = 4 * U32 * np.sqrt(d) * mag
         acc += (_flip_risk(x2r, rel) * _ulp(x2r)).astype(np.float32) @ Wgu.T
-        gu = (x2.astype(np.float32) @ np.asarray(tw[f"layers.{l}.wgate_up"], np.float32).T).astype(np.float64)
+        acc = acc * rs + (2.0 ** -18 + rel_rs) * mag * rs
+        gu = (x2.astype(np.float32) @ np.asarray(tw[f"layers.{l}.wgate_up"], np.float32).T).astype(np.float64) * rs
         gg, uu = gu[:, :f], gu[:, f:]
         sg = 1.0 / (1.0 + np.exp(-gg))
         dsilu = sg * (1.0 + gg * (1.0 - sg))

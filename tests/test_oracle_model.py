@@ -119,6 +119,36 @@ def test_head_permutation_invariance():
     np.testing.assert_allclose(a, b, rtol=1e-11, atol=1e-11)
 
 
+def test_unrounded_layer_is_the_textbook_prenorm_block():
+    """With the rounding points off, the layer functions (norm scale applied after the projection)
+    equal the textbook LLaMA block written with torch's own rms_norm and silu: RMSNorm, then the
+    QKV projection and RoPE; residual + O projection, RMSNorm, gate/up, SiLU(gate) * up."""
+    from oracle.model import _layer_mlp_act, _layer_pre_attn
+    from oracle.numerics import rope
+    m = _model(rnd=False)
+    sp = SPEC
+    d, H, hd, f = sp.d_model, sp.n_heads, sp.head_dim, sp.d_ffn
+    rng = np.random.default_rng(5)
+    h = rng.standard_normal((6, d)) * 3.0
+    pos = np.arange(6) + 4
+    th = torch.from_numpy
+    for l in range(sp.n_layers):
+        x = torch.nn.functional.rms_norm(th(h), (d,), th(m.W(f"layers.{l}.attn_norm")), eps=sp.rms_eps).numpy()
+        qkv = x @ m.W(f"layers.{l}.wqkv").T
+        q, k, v = _layer_pre_attn(m, l, h, pos)
+        np.testing.assert_allclose(q, rope(qkv[:, :d].reshape(-1, H, hd), pos, sp.rope_theta), rtol=1e-10, atol=1e-12)
+        np.testing.assert_allclose(k, rope(qkv[:, d:2 * d].reshape(-1, H, hd), pos, sp.rope_theta), rtol=1e-10, atol=1e-12)
+        np.testing.assert_allclose(v, qkv[:, 2 * d:].reshape(-1, H, hd), rtol=1e-10, atol=1e-12)
+        o = rng.standard_normal((6, d))
+        h2 = h + o @ m.W(f"layers.{l}.wo").T
+        x2 = torch.nn.functional.rms_norm(th(h2), (d,), th(m.W(f"layers.{l}.mlp_norm")), eps=sp.rms_eps)
+        gu = x2 @ th(m.W(f"layers.{l}.wgate_up")).T
+        act = (torch.nn.functional.silu(gu[:, :f]) * gu[:, f:]).numpy()
+        h_out, a = _layer_mlp_act(m, l, h, o)
+        np.testing.assert_allclose(h_out, h2, rtol=1e-12, atol=1e-12)
+        np.testing.assert_allclose(a, act, rtol=1e-10, atol=1e-12)
+
+
 def test_rounding_points_are_bf16():
     m = _model()
     from oracle.model import _layer_pre_attn

@@ -6,7 +6,7 @@ import numpy as np
 import pytest
 import torch
 
-from oracle.numerics import bf16, rmsnorm, rope, silu
+from oracle.numerics import bf16, rms_scale, rmsnorm, rope, silu
 from oracle.philox import (draw_u32, gumbel, philox4x32_10, u_accept, u_open)
 
 GOLD = os.path.join(os.path.dirname(__file__), "golden")
@@ -35,6 +35,15 @@ def test_rmsnorm_closed_form():
     x = np.random.default_rng(1).standard_normal((5, 32))
     ref = torch.nn.functional.rms_norm(torch.from_numpy(x), (32,), torch.from_numpy(g[:32]), eps=1e-6).numpy()
     np.testing.assert_allclose(rmsnorm(x, g[:32], 1e-6), ref, rtol=1e-12)
+
+
+def test_rms_scale_closed_form():
+    """RMSNorm's per-row scale alone: exact values, and times h it is torch's gain-free rms_norm."""
+    np.testing.assert_array_equal(rms_scale(np.array([[2.0, -2.0], [1.0, 1.0]]), 0.0), [[0.5], [1.0]])
+    np.testing.assert_allclose(rms_scale(np.array([[3.0, 4.0]]), 0.0), [[1.0 / np.sqrt(12.5)]], rtol=1e-15)
+    x = np.random.default_rng(2).standard_normal((4, 48))
+    ref = torch.nn.functional.rms_norm(torch.from_numpy(x), (48,), None, eps=1e-6).numpy()
+    np.testing.assert_allclose(x * rms_scale(x, 1e-6), ref, rtol=1e-12)
 
 
 def test_rope_identity_norm_and_relative_position():
