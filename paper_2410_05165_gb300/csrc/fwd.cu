@@ -45,6 +45,7 @@ constexpr int kRegsLaunch = 168, kRegsRoles = 80, kRegsCompute = 208;
 static_assert(128 * kRegsRoles + 256 * kRegsCompute <= FWD_THREADS * kRegsLaunch, "register split over the launch's total");
 static_assert(32 * (kRegsRoles + 2 * kRegsCompute) <= 16384, "register split over a sub-partition's file");
 static_assert(kRegsRoles % 8 == 0 && kRegsCompute % 8 == 0 && kRegsRoles >= 24 && kRegsCompute <= 256, "setmaxnreg range");
+constexpr int RED_PB = 3;             // split parts in flight in a chunk's sum
 constexpr int ITEM_ROWS_FWD = 1024;   // item-code rows of the LM head (4 levels x 256 codes)
 
 template <int BN>
@@ -155,6 +156,17 @@ __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* a) {
   unsigned v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(a) : "memory");
   return v;
+}
+// Publishing a CTA's split parts: every thread stores, the CTA synchronises, then one thread's
+// release (or acquire-release) add at gpu scope makes all of those stores visible to whoever
+// acquires the counter (and synchronises its own CTA after that).
+__device__ __forceinline__ void red_release_add(int* a, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(a), "r"(v) : "memory");
+}
+__device__ __forceinline__ int atom_acq_rel_add(int* a, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(a), "r"(v) : "memory");
+  return old;
 }
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 
@@ -466,11 +478,11 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
       if (lane == 0) mbar_arrive(&tempty[acc]);
       sk_tile[nsk++] = tile;
     }
-    __threadfence();
     named_bar_sync(1, CT);
     int* skc = p.sk_counters + (size_t)gi * G;
     if (ctid == 0)
-      for (int j = 0; j < nsk; ++j) atomicAdd(&skc[sk_tile[j]], 1);
+      for (int j = 0; j < nsk; ++j) red_release_add(&skc[sk_tile[j]], 1);
+    if (p.trace && ctid == 0) p.trace[((size_t)5 * NP + ph) * G + c] = globaltimer_ns();
     for (int j = 0; j < nsk; ++j) {
       const int t = sk_tile[j];
       const long long tu0 = (long long)t * kb;
@@ -482,14 +494,30 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
       if (ctid == 0) *flag = counter_wait(&skc[t], parts, p.err) ? 1 : 0;
       named_bar_sync(1, CT);
       if (!*flag) return false;
+      const bool tr_on = p.trace && ctid == 0 && j == 0;
+      if (tr_on) p.trace[((size_t)6 * NP + ph) * G + c] = globaltimer_ns();
       const int nch = min(BN / 32, (g.rows - n_tile * BN + 31) / 32);
+      if (g.dh_out) {
+        // residual updates: both warpgroups on each chunk of this part, 16 tokens each
+        for (int ch = c - c_first; ch < nch; ch += parts) {
+          if (ch * 32 + 16 * wg >= g.rows - n_tile * BN) continue;   // (warpgroup-uniform)
+          ws_reduce_resnorm_half<RED_PB>(ea, p.ws, part_slot, parts, ch, wg, m_tile, n_tile * BN + ch * 32, wt, staging,
+                                         wbar);
+          named_bar_sync(wbar, 128);
+          if (tr_on) p.trace[((size_t)9 * NP + ph) * G + c] = globaltimer_ns();
+        }
+        named_bar_sync(1, CT);   // flag, part_slot and the token tables are reused
+        continue;
+      }
       int k = 0;
       for (int ch = c - c_first; ch < nch; ch += parts, ++k) {
         if ((k & 1) != wg) continue;
         ws_reduce_chunk<1>(p.ws, part_slot, parts, ch, m, staging);
         named_bar_sync(wbar, 128);
+        if (tr_on && k == 0) p.trace[((size_t)8 * NP + ph) * G + c] = globaltimer_ns();
         epi_dispatch<BN>(g.epi, s_ea, staging, m_tile, n_tile, ch, wt, tpos, tkvr, trs_e, wbar);
         named_bar_sync(wbar, 128);
+        if (tr_on && k == 0) p.trace[((size_t)9 * NP + ph) * G + c] = globaltimer_ns();
       }
       named_bar_sync(1, CT);   // flag, part_slot and the token tables are reused
     }
@@ -558,11 +586,10 @@ __device__ __forceinline__ bool gemm_epi_phase(const FwdParams& p, int gi, int p
     ws_store_partial(p.ws + slot * GEMM_WS_SLOT_FLOATS, tb, nch, m, wg, 2);
     tc_fence_before();
     if (lane == 0) mbar_arrive(&tempty[acc]);
-    __threadfence();
     named_bar_sync(1, CT);
     if (p.trace && ctid == 0) p.trace[((size_t)5 * NP + ph) * G + c] = globaltimer_ns();
     if (ctid == 0) {
-      const int old = atomicAdd(&p.counters[tile], 1);
+      const int old = atom_acq_rel_add(&p.counters[tile], 1);
       const int last = (old == parts - 1);
       if (last) {
         p.counters[tile] = 0;

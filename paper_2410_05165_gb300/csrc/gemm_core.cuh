@@ -169,40 +169,114 @@ __device__ __forceinline__ void load_norm_scales(const GemmArgs& a, int n_tile, 
   }
 }
 
-// EPI_RESNORM over one 32-token chunk (O / down projections): h += product (fp32 residual,
-// read-modify-write; every (row, token) belongs to one chunk of one CTA), xg = bf16(g * h) for the
-// next GEMM, and the partial sums of squares of the updated rows.  128 threads (ep_tid = the tile
-// row they own); `bar` is a named barrier of those 128 threads.  st (staging, [32 tokens][128 rows])
-// holds the product and is overwritten with the updated residual.
-__device__ __forceinline__ void epi_resnorm(const GemmArgs& a, float* st, int m_tile, int tok0, int ep_tid, int bar) {
-  const int nv = min(32, a.T - tok0);
+// Partial sums of squares of the updated residual of tokens j0 .. j0 + NJ - 1 of a chunk (st holds
+// them, [token][128 rows]), nv of them valid: 4 threads per token (warps 0 .. NJ / 8 - 1), token jj
+// of the range, quarter sub of the rows; the rotation follows the token's index mod 32 and also
+// spreads a warp's shared-memory reads over the 32 banks.
+template <int NJ>
+__device__ __forceinline__ void resnorm_ssq(const GemmArgs& a, const float* st, int m_tile, int tok0, int j0, int nv,
+                                            int ep_tid) {
+  if (ep_tid < 4 * NJ) {
+    const int jj = ep_tid >> 2, sub = ep_tid & 3, j = j0 + jj;
+    const float* sj = st + j * GEMM_BM + sub * 32;
+    float s = ssq32([&](int r) { return sj[r]; }, ssq_rot(sub, j));
+    s += __shfl_xor_sync(0xffffffffu, s, 1);
+    s += __shfl_xor_sync(0xffffffffu, s, 2);
+    if (sub == 0 && jj < nv) a.ssq_out[(size_t)m_tile * a.ssq_ld + tok0 + j] = s;
+  }
+}
+
+// EPI_RESNORM over tokens j0 .. j0 + NJ - 1 of one 32-token chunk (O / down projections): h +=
+// product (fp32 residual, read-modify-write; every (row, token) belongs to one chunk of one CTA),
+// xg = bf16(g * h) for the next GEMM, and the partial sums of squares of the updated rows.  128
+// threads (ep_tid = the tile row they own); `bar` is a named barrier of those 128 threads.  st
+// (staging, [32 tokens][128 rows]) holds the product in the rows of those tokens and is overwritten
+// there with the updated residual.  The arithmetic per token does not depend on NJ or j0.
+template <int NJ = 32>
+__device__ __forceinline__ void epi_resnorm(const GemmArgs& a, float* st, int m_tile, int tok0, int ep_tid, int bar,
+                                            int j0 = 0) {
+  const int nv = min(NJ, a.T - tok0 - j0);   // valid tokens of the range
   const int m = ep_tid, row = m_tile * GEMM_BM + m;
   const bool in = row < a.M;
-  float* base = a.out_f32 + (size_t)tok0 * a.ldo + row;
+  float* base = a.out_f32 + (size_t)(tok0 + j0) * a.ldo + row;
+  float* sb = st + j0 * GEMM_BM;
   const bool xg = a.gain != nullptr;
   const float g = (in && xg) ? __bfloat162float(a.gain[row]) : 0.f;
-  float old[32];
+  float old[NJ];
 #pragma unroll
-  for (int n = 0; n < 32; ++n) old[n] = (in && n < nv) ? __ldcg(base + (size_t)n * a.ldo) : 0.f;
+  for (int n = 0; n < NJ; ++n) old[n] = (in && n < nv) ? __ldcg(base + (size_t)n * a.ldo) : 0.f;
 #pragma unroll
-  for (int n = 0; n < 32; ++n) {
-    const float v = in ? old[n] + st[n * GEMM_BM + m] : 0.f;
+  for (int n = 0; n < NJ; ++n) {
+    const float v = in ? old[n] + sb[n * GEMM_BM + m] : 0.f;
     if (in && n < nv) {
       base[(size_t)n * a.ldo] = v;
-      if (xg) a.xg_out[(size_t)(tok0 + n) * a.ldo + row] = __float2bfloat16_rn(v * g);
+      if (xg) a.xg_out[(size_t)(tok0 + j0 + n) * a.ldo + row] = __float2bfloat16_rn(v * g);
     }
-    st[n * GEMM_BM + m] = v;
+    sb[n * GEMM_BM + m] = v;
   }
   if (a.ssq_out == nullptr) return;
   named_bar_sync(bar, 128);
-  // token j of the chunk (j = its index mod 32), quarter sub of the rows; the rotation also spreads
-  // a warp's shared-memory reads over the 32 banks
-  const int j = ep_tid >> 2, sub = ep_tid & 3;
-  const float* sj = st + j * GEMM_BM + sub * 32;
-  float s = ssq32([&](int r) { return sj[r]; }, ssq_rot(sub, j));
-  s += __shfl_xor_sync(0xffffffffu, s, 1);
-  s += __shfl_xor_sync(0xffffffffu, s, 2);
-  if (sub == 0 && j < nv) a.ssq_out[(size_t)m_tile * a.ssq_ld + tok0 + j] = s;
+  resnorm_ssq<NJ>(a, st, m_tile, tok0, j0, nv, ep_tid);
+}
+
+// Split-K sum (in k order, from zero) of tokens 16 half .. 16 half + 15 of chunk ch of the parts in
+// `slot`, then EPI_RESNORM of those tokens: epi_resnorm<16>'s arithmetic, with the residual loads
+// issued together with the first parts' loads.  PB parts in flight at once.
+template <int PB>
+__device__ __forceinline__ void ws_reduce_resnorm_half(const GemmArgs& a, const float* ws, const int* slot, int parts,
+                                                       int ch, int half, int m_tile, int tok0, int ep_tid,
+                                                       float* st, int bar) {
+  const int j0 = 16 * half;
+  const int nv = min(16, a.T - tok0 - j0);
+  const int m = ep_tid, row = m_tile * GEMM_BM + m;
+  const bool in = row < a.M;
+  float* base = a.out_f32 + (size_t)(tok0 + j0) * a.ldo + row;
+  float old[16], acc[16];
+#pragma unroll
+  for (int n = 0; n < 16; ++n) {
+    old[n] = (in && n < nv) ? __ldcg(base + (size_t)n * a.ldo) : 0.f;
+    acc[n] = 0.f;
+  }
+  const float4* w4 = reinterpret_cast<const float4*>(ws);
+  constexpr long long SLOT4 = GEMM_WS_SLOT_FLOATS / 4;
+  for (int p0 = 0; p0 < parts; p0 += PB) {
+    float4 v[PB][4];
+#pragma unroll
+    for (int b = 0; b < PB; ++b) {
+      if (p0 + b < parts) {
+        const float4* src = w4 + (long long)slot[p0 + b] * SLOT4 + (ch * 8 + 4 * half) * GEMM_BM + m;
+#pragma unroll
+        for (int j4 = 0; j4 < 4; ++j4) v[b][j4] = __ldcg(src + j4 * GEMM_BM);
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < PB; ++b) {
+      if (p0 + b < parts) {
+#pragma unroll
+        for (int j4 = 0; j4 < 4; ++j4) {
+          acc[4 * j4] += v[b][j4].x;
+          acc[4 * j4 + 1] += v[b][j4].y;
+          acc[4 * j4 + 2] += v[b][j4].z;
+          acc[4 * j4 + 3] += v[b][j4].w;
+        }
+      }
+    }
+  }
+  const bool xg = a.gain != nullptr;
+  const float g = (in && xg) ? __bfloat162float(a.gain[row]) : 0.f;
+  float* sb = st + j0 * GEMM_BM;
+#pragma unroll
+  for (int n = 0; n < 16; ++n) {
+    const float vv = in ? old[n] + acc[n] : 0.f;
+    if (in && n < nv) {
+      base[(size_t)n * a.ldo] = vv;
+      if (xg) a.xg_out[(size_t)(tok0 + j0 + n) * a.ldo + row] = __float2bfloat16_rn(vv * g);
+    }
+    sb[n * GEMM_BM + m] = vv;
+  }
+  if (a.ssq_out == nullptr) return;
+  named_bar_sync(bar, 128);
+  resnorm_ssq<16>(a, st, m_tile, tok0, j0, nv, ep_tid);
 }
 
 // st: staging [32 tokens][128 rows] fp32 of one chunk; 128 threads (ep_tid) write the outputs.
