@@ -134,10 +134,10 @@ __device__ __forceinline__ void load_tok_tables(const GemmArgs& a, int n_tile, i
 // ---- RMSNorm folded into the GEMMs around it
 // Sum of squares of 32 values v(0 .. 31) in the rotated order rot, rot + 1, ... (mod 32), one fused
 // multiply-add per value.  A token's partial sum over a 128-row tile of the residual is
-// (q0 + q1) + (q2 + q3), q_s = ssq32 over rows 32 s .. 32 s + 31 of the tile with rot =
-// ssq_rot(s, token); rows past d count as zero.  Every producer of partial sums (the O / down
-// epilogue, the embedding rows) uses exactly these orders, so a token's sums do not depend on the
-// kernel or the schedule that made them.
+// (q0 + q1) + (q2 + q3), q_s = ssq32 over rows 32 s .. 32 s + 31 of the tile with rot = ssq_rot(s);
+// rows past d count as zero.  Every producer of partial sums (the O / down epilogue, the embedding
+// rows) uses exactly these orders, and none depends on the token's index in the call, so a token's
+// sums depend neither on the kernel or schedule that made them nor on the other tokens of the call.
 template <class F>
 __device__ __forceinline__ float ssq32(F v, int rot) {
   float s = 0.f;
@@ -148,7 +148,8 @@ __device__ __forceinline__ float ssq32(F v, int rot) {
   }
   return s;
 }
-__device__ __forceinline__ int ssq_rot(int sub, int tok) { return (sub * 8 + (tok & 31)) & 31; }
+// (the four quarters start on different banks of the staging rows)
+__device__ __forceinline__ int ssq_rot(int sub) { return sub * 8; }
 
 // 1 / rms of token t (RMSNorm's per-token scale) from its partial sums, added in tile order.
 __device__ __forceinline__ float norm_scale(const float* ssq, int ld, int d, float eps, int t) {
@@ -171,15 +172,14 @@ __device__ __forceinline__ void load_norm_scales(const GemmArgs& a, int n_tile, 
 
 // Partial sums of squares of the updated residual of tokens j0 .. j0 + NJ - 1 of a chunk (st holds
 // them, [token][128 rows]), nv of them valid: 4 threads per token (warps 0 .. NJ / 8 - 1), token jj
-// of the range, quarter sub of the rows; the rotation follows the token's index mod 32 and also
-// spreads a warp's shared-memory reads over the 32 banks.
+// of the range, quarter sub of the rows.
 template <int NJ>
 __device__ __forceinline__ void resnorm_ssq(const GemmArgs& a, const float* st, int m_tile, int tok0, int j0, int nv,
                                             int ep_tid) {
   if (ep_tid < 4 * NJ) {
     const int jj = ep_tid >> 2, sub = ep_tid & 3, j = j0 + jj;
     const float* sj = st + j * GEMM_BM + sub * 32;
-    float s = ssq32([&](int r) { return sj[r]; }, ssq_rot(sub, j));
+    float s = ssq32([&](int r) { return sj[r]; }, ssq_rot(sub));
     s += __shfl_xor_sync(0xffffffffu, s, 1);
     s += __shfl_xor_sync(0xffffffffu, s, 2);
     if (sub == 0 && jj < nv) a.ssq_out[(size_t)m_tile * a.ssq_ld + tok0 + j] = s;

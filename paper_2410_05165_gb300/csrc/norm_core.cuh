@@ -67,7 +67,7 @@ __device__ __forceinline__ void embed_row(const __nv_bfloat16* er, const __nv_bf
     const int mt = qi >> 2, sub = qi & 3;
     const int r0 = mt * GEMM_BM + sub * 32;
     float s = 0.f;
-    if (qi < nq) s = ssq32([&](int r) { return r0 + r < d ? __bfloat162float(er[r0 + r]) : 0.f; }, ssq_rot(sub, t));
+    if (qi < nq) s = ssq32([&](int r) { return r0 + r < d ? __bfloat162float(er[r0 + r]) : 0.f; }, ssq_rot(sub));
     s += __shfl_xor_sync(0xffffffffu, s, 1);
     s += __shfl_xor_sync(0xffffffffu, s, 2);
     if (qi < nq && sub == 0) ssq[(size_t)mt * ld + t] = s;

@@ -413,6 +413,37 @@ def test_persistent_forward_equals_per_op_multi_user(ats, cfg, layers, B, monkey
     np.testing.assert_array_equal(outs[0], outs[1])
 
 
+@pytest.mark.parametrize("mode", ["per_op", "persistent"])
+def test_identical_users_get_identical_logits(ats, mode, monkeypatch):
+    """Three users with the same 40-token history and the same drafted tree in one call (the prefill's
+    120 tokens and the verification's 90 tree tokens each fit one 128-token tile, so every token
+    sees the same split-K partition): every node's logits are the same for all three, bit for bit,
+    although their tokens sit at different rows of the call -- no per-token arithmetic (norm sums,
+    split-K sums, attention) depends on a token's index or on the other tokens."""
+    monkeypatch.setenv("ATSPEED_FORWARD", mode)
+    w = synth.workload("mid")
+    spec = synth.ModelSpec(2, w.target.d_model, w.target.n_heads, w.target.d_ffn, w.target.vocab)
+    items = synth.make_items(5000, w.code_dist, w.zipf_a, w.seed)
+    prompt = synth.make_prompts(1, w.prompt_len, spec.vocab, w.seed)[0][:40]
+    B, K, N, G = 3, 5, 10, 3
+    _, levels = synth.random_tree(items, 0, 1, G, N, seed=17)
+    cnt1, par1, cod1, sq1 = _tree_arrays(levels, 1, G, N)
+    cnt, par, cod, sq = (np.repeat(a, B, axis=0) for a in (cnt1, par1, cod1, sq1))
+    ctx = _ctx(ats, spec, None, items, w.code_base, B, len(prompt), K, N, G, seed=w.seed)
+    _prefill(ats, ctx, [prompt] * B)
+    o = ats.opts(K, N, G)
+    ctx.begin_step(o)
+    ctx.set_tree(cnt, par, cod, sq)
+    ctx.verify(o, ats.STRICT)
+    got = [np.stack([ctx.node_logits(0, u, 0)] +
+                    [ctx.node_logits(0, u, K + j * N + k) for j, lvl in enumerate(levels) for k in range(len(lvl))])
+           for u in range(B)]
+    ctx.close()
+    assert np.all(np.isfinite(got[0]))
+    for u in range(1, B):
+        np.testing.assert_array_equal(got[u], got[0])
+
+
 # ------------------------------------------------------------------------------------------------
 # FULL normalisation (whole-vocabulary log-softmax, then the trie mask)
 # ------------------------------------------------------------------------------------------------
