@@ -186,6 +186,42 @@ __device__ __forceinline__ void resnorm_ssq(const GemmArgs& a, const float* st, 
   }
 }
 
+// The updated residual of tokens j0 .. j0 + NJ - 1 of a chunk (st, [token][128 rows]; nv of them
+// valid) to h and bf16(g * h) to xg: a thread stores four adjacent rows (one 16-byte h store, one
+// 8-byte xg store per token), warp w the tokens j0 + w NJ / 4 .., so a warp's store covers a token's
+// 128 rows in one piece.  (M, the residual's width, is a multiple of 4.)
+template <int NJ>
+__device__ __forceinline__ void resnorm_store(const GemmArgs& a, const float* st, int m_tile, int tok0, int j0, int nv,
+                                              int ep_tid) {
+  constexpr int TPW = NJ / 4;   // tokens per warp
+  const int rq = ep_tid & 31, w = ep_tid >> 5;
+  const int row = m_tile * GEMM_BM + 4 * rq;
+  if (row >= a.M) return;
+  const bool xg = a.gain != nullptr;
+  float2 g01 = make_float2(0.f, 0.f), g23 = g01;
+  if (xg) {
+    const uint2 graw = *reinterpret_cast<const uint2*>(a.gain + row);
+    const __nv_bfloat162* gb = reinterpret_cast<const __nv_bfloat162*>(&graw);
+    g01 = __bfloat1622float2(gb[0]);
+    g23 = __bfloat1622float2(gb[1]);
+  }
+#pragma unroll
+  for (int k = 0; k < TPW; ++k) {
+    const int n = w * TPW + k;
+    if (n < nv) {
+      const float4 v = *reinterpret_cast<const float4*>(st + (j0 + n) * GEMM_BM + 4 * rq);
+      const size_t e = (size_t)(tok0 + j0 + n) * a.ldo + row;
+      *reinterpret_cast<float4*>(a.out_f32 + e) = v;
+      if (xg) {
+        __nv_bfloat162 o[2];
+        o[0] = __floats2bfloat162_rn(v.x * g01.x, v.y * g01.y);
+        o[1] = __floats2bfloat162_rn(v.z * g23.x, v.w * g23.y);
+        *reinterpret_cast<uint2*>(a.xg_out + e) = *reinterpret_cast<const uint2*>(o);
+      }
+    }
+  }
+}
+
 // EPI_RESNORM over tokens j0 .. j0 + NJ - 1 of one 32-token chunk (O / down projections): h +=
 // product (fp32 residual, read-modify-write; every (row, token) belongs to one chunk of one CTA),
 // xg = bf16(g * h) for the next GEMM, and the partial sums of squares of the updated rows.  128
@@ -198,25 +234,17 @@ __device__ __forceinline__ void epi_resnorm(const GemmArgs& a, float* st, int m_
   const int nv = min(NJ, a.T - tok0 - j0);   // valid tokens of the range
   const int m = ep_tid, row = m_tile * GEMM_BM + m;
   const bool in = row < a.M;
-  float* base = a.out_f32 + (size_t)(tok0 + j0) * a.ldo + row;
+  const float* base = a.out_f32 + (size_t)(tok0 + j0) * a.ldo + row;
   float* sb = st + j0 * GEMM_BM;
-  const bool xg = a.gain != nullptr;
-  const float g = (in && xg) ? __bfloat162float(a.gain[row]) : 0.f;
   float old[NJ];
 #pragma unroll
   for (int n = 0; n < NJ; ++n) old[n] = (in && n < nv) ? __ldcg(base + (size_t)n * a.ldo) : 0.f;
 #pragma unroll
-  for (int n = 0; n < NJ; ++n) {
-    const float v = in ? old[n] + sb[n * GEMM_BM + m] : 0.f;
-    if (in && n < nv) {
-      base[(size_t)n * a.ldo] = v;
-      if (xg) a.xg_out[(size_t)(tok0 + j0 + n) * a.ldo + row] = __float2bfloat16_rn(v * g);
-    }
-    sb[n * GEMM_BM + m] = v;
-  }
-  if (a.ssq_out == nullptr) return;
+  for (int n = 0; n < NJ; ++n) sb[n * GEMM_BM + m] = in ? old[n] + sb[n * GEMM_BM + m] : 0.f;
+  // the sums of squares before the stores (their shared-memory reads would queue behind them)
   named_bar_sync(bar, 128);
-  resnorm_ssq<NJ>(a, st, m_tile, tok0, j0, nv, ep_tid);
+  if (a.ssq_out != nullptr) resnorm_ssq<NJ>(a, st, m_tile, tok0, j0, nv, ep_tid);
+  resnorm_store<NJ>(a, st, m_tile, tok0, j0, nv, ep_tid);
 }
 
 // Split-K sum (in k order, from zero) of tokens 16 half .. 16 half + 15 of chunk ch of the parts in
@@ -230,7 +258,7 @@ __device__ __forceinline__ void ws_reduce_resnorm_half(const GemmArgs& a, const 
   const int nv = min(16, a.T - tok0 - j0);
   const int m = ep_tid, row = m_tile * GEMM_BM + m;
   const bool in = row < a.M;
-  float* base = a.out_f32 + (size_t)(tok0 + j0) * a.ldo + row;
+  const float* base = a.out_f32 + (size_t)(tok0 + j0) * a.ldo + row;
   float old[16], acc[16];
 #pragma unroll
   for (int n = 0; n < 16; ++n) {
@@ -262,21 +290,12 @@ __device__ __forceinline__ void ws_reduce_resnorm_half(const GemmArgs& a, const 
       }
     }
   }
-  const bool xg = a.gain != nullptr;
-  const float g = (in && xg) ? __bfloat162float(a.gain[row]) : 0.f;
   float* sb = st + j0 * GEMM_BM;
 #pragma unroll
-  for (int n = 0; n < 16; ++n) {
-    const float vv = in ? old[n] + acc[n] : 0.f;
-    if (in && n < nv) {
-      base[(size_t)n * a.ldo] = vv;
-      if (xg) a.xg_out[(size_t)(tok0 + j0 + n) * a.ldo + row] = __float2bfloat16_rn(vv * g);
-    }
-    sb[n * GEMM_BM + m] = vv;
-  }
-  if (a.ssq_out == nullptr) return;
+  for (int n = 0; n < 16; ++n) sb[n * GEMM_BM + m] = in ? old[n] + acc[n] : 0.f;
   named_bar_sync(bar, 128);
-  resnorm_ssq<16>(a, st, m_tile, tok0, j0, nv, ep_tid);
+  if (a.ssq_out != nullptr) resnorm_ssq<16>(a, st, m_tile, tok0, j0, nv, ep_tid);
+  resnorm_store<16>(a, st, m_tile, tok0, j0, nv, ep_tid);
 }
 
 // st: staging [32 tokens][128 rows] fp32 of one chunk; 128 threads (ep_tid) write the outputs.
