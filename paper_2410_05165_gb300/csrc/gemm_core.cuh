@@ -140,12 +140,12 @@ __device__ __forceinline__ void load_tok_tables(const GemmArgs& a, int n_tile, i
 // sums depend neither on the kernel or schedule that made them nor on the other tokens of the call.
 template <class F>
 __device__ __forceinline__ float ssq32(F v, int rot) {
+  float x[32];   // every value loaded first, then the dependent chain
+#pragma unroll
+  for (int i = 0; i < 32; ++i) x[i] = v((i + rot) & 31);
   float s = 0.f;
-#pragma unroll 8
-  for (int i = 0; i < 32; ++i) {
-    const float x = v((i + rot) & 31);
-    s = __fmaf_rn(x, x, s);
-  }
+#pragma unroll
+  for (int i = 0; i < 32; ++i) s = __fmaf_rn(x[i], x[i], s);
   return s;
 }
 // (the four quarters start on different banks of the staging rows)
@@ -173,12 +173,14 @@ __device__ __forceinline__ void load_norm_scales(const GemmArgs& a, int n_tile, 
 // Partial sums of squares of the updated residual of tokens j0 .. j0 + NJ - 1 of a chunk (st holds
 // them, [token][128 rows]), nv of them valid: 4 threads per token (warps 0 .. NJ / 8 - 1), token jj
 // of the range, quarter sub of the rows.
-template <int NJ>
-__device__ __forceinline__ void resnorm_ssq(const GemmArgs& a, const float* st, int m_tile, int tok0, int j0, int nv,
+// sr: the first of those tokens' rows, SR floats apart (the order of the sums does not depend on
+// where the rows sit: a row stride of 132 spreads a warp's eight tokens over the banks).
+template <int NJ, int SR = GEMM_BM>
+__device__ __forceinline__ void resnorm_ssq(const GemmArgs& a, const float* sr, int m_tile, int tok0, int j0, int nv,
                                             int ep_tid) {
   if (ep_tid < 4 * NJ) {
     const int jj = ep_tid >> 2, sub = ep_tid & 3, j = j0 + jj;
-    const float* sj = st + j * GEMM_BM + sub * 32;
+    const float* sj = sr + jj * SR + sub * 32;
     float s = ssq32([&](int r) { return sj[r]; }, ssq_rot(sub));
     s += __shfl_xor_sync(0xffffffffu, s, 1);
     s += __shfl_xor_sync(0xffffffffu, s, 2);
@@ -190,8 +192,8 @@ __device__ __forceinline__ void resnorm_ssq(const GemmArgs& a, const float* st, 
 // valid) to h and bf16(g * h) to xg: a thread stores four adjacent rows (one 16-byte h store, one
 // 8-byte xg store per token), warp w the tokens j0 + w NJ / 4 .., so a warp's store covers a token's
 // 128 rows in one piece.  (M, the residual's width, is a multiple of 4.)
-template <int NJ>
-__device__ __forceinline__ void resnorm_store(const GemmArgs& a, const float* st, int m_tile, int tok0, int j0, int nv,
+template <int NJ, int SR = GEMM_BM>
+__device__ __forceinline__ void resnorm_store(const GemmArgs& a, const float* sr, int m_tile, int tok0, int j0, int nv,
                                               int ep_tid) {
   constexpr int TPW = NJ / 4;   // tokens per warp
   const int rq = ep_tid & 31, w = ep_tid >> 5;
@@ -209,7 +211,7 @@ __device__ __forceinline__ void resnorm_store(const GemmArgs& a, const float* st
   for (int k = 0; k < TPW; ++k) {
     const int n = w * TPW + k;
     if (n < nv) {
-      const float4 v = *reinterpret_cast<const float4*>(st + (j0 + n) * GEMM_BM + 4 * rq);
+      const float4 v = *reinterpret_cast<const float4*>(sr + n * SR + 4 * rq);
       const size_t e = (size_t)(tok0 + j0 + n) * a.ldo + row;
       *reinterpret_cast<float4*>(a.out_f32 + e) = v;
       if (xg) {
@@ -243,8 +245,8 @@ __device__ __forceinline__ void epi_resnorm(const GemmArgs& a, float* st, int m_
   for (int n = 0; n < NJ; ++n) sb[n * GEMM_BM + m] = in ? old[n] + sb[n * GEMM_BM + m] : 0.f;
   // the sums of squares before the stores (their shared-memory reads would queue behind them)
   named_bar_sync(bar, 128);
-  if (a.ssq_out != nullptr) resnorm_ssq<NJ>(a, st, m_tile, tok0, j0, nv, ep_tid);
-  resnorm_store<NJ>(a, st, m_tile, tok0, j0, nv, ep_tid);
+  if (a.ssq_out != nullptr) resnorm_ssq<NJ>(a, sb, m_tile, tok0, j0, nv, ep_tid);
+  resnorm_store<NJ>(a, sb, m_tile, tok0, j0, nv, ep_tid);
 }
 
 // Split-K sum (in k order, from zero) of tokens 16 half .. 16 half + 15 of chunk ch of the parts in
@@ -290,12 +292,14 @@ __device__ __forceinline__ void ws_reduce_resnorm_half(const GemmArgs& a, const 
       }
     }
   }
-  float* sb = st + j0 * GEMM_BM;
+  // the updated rows go to the start of st, 132 floats apart (16 x 132 floats fit the 32 x 128 of a
+  // staging buffer; float4-aligned rows; conflict-free sums of squares)
+  constexpr int SR = GEMM_BM + 4;
 #pragma unroll
-  for (int n = 0; n < 16; ++n) sb[n * GEMM_BM + m] = in ? old[n] + acc[n] : 0.f;
+  for (int n = 0; n < 16; ++n) st[n * SR + m] = in ? old[n] + acc[n] : 0.f;
   named_bar_sync(bar, 128);
-  if (a.ssq_out != nullptr) resnorm_ssq<16>(a, st, m_tile, tok0, j0, nv, ep_tid);
-  resnorm_store<16>(a, st, m_tile, tok0, j0, nv, ep_tid);
+  if (a.ssq_out != nullptr) resnorm_ssq<16, SR>(a, st, m_tile, tok0, j0, nv, ep_tid);
+  resnorm_store<16, SR>(a, st, m_tile, tok0, j0, nv, ep_tid);
 }
 
 // st: staging [32 tokens][128 rows] fp32 of one chunk; 128 threads (ep_tid) write the outputs.
