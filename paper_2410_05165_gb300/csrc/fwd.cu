@@ -6,18 +6,19 @@
 // folded into the GEMMs around them (x = h / rms(h) * g, and W x = (W (g h)) / rms(h)): the O /
 // down epilogue adds its product to h and leaves bf16(g h) and per-128-row-tile sums of squares of
 // h; the QKV / gate-up epilogue multiplies each token's product by 1 / rms(h) from those sums.  (The
-// program keeps the index slots of the two norm phases per layer, 7 per layer, for the trace.)  The GEMM phases reuse the stream-K decomposition of the
-// standalone GEMM (equal contiguous ranges of (tile, k-block) units per CTA, split tiles reduced
-// by their last CTA), but their operands flow through two rings that live for the whole launch:
+// program keeps the index slots of the two folded norm phases per layer, 7 per layer, for the
+// trace.)  The GEMM phases reuse the stream-K decomposition of the standalone GEMM (whole tiles
+// and stream-K units per CTA, split tiles summed in k order), but their operands flow through two
+// rings that live for the whole launch:
 //   * the weight ring (A, 16 KB per stage) is filled by a producer warp that walks every GEMM
 //     phase of the forward in order and never waits for a grid barrier -- weights do not depend
-//     on activations -- so HBM keeps streaming the next phase's weights during barriers, norms
-//     and attention;
+//     on activations -- so HBM keeps streaming the next phase's weights during barriers, split-sum
+//     tails and attention;
 //   * the activation ring (B) is filled by a second producer warp that waits for the barrier that
 //     publishes the phase's input.
 // Warp roles (384 threads): 0 weight TMA, 1 activation TMA, 2 TMEM + MMA issue, 3 idle; 4..11 two
 // compute warpgroups (GEMM epilogues -- a warp reads the TMEM lane quadrant of its id mod 4 --,
-// RMSNorm rows, tree attention).
+// the embedding and final-norm rows, tree attention).
 // Every wait is bounded; a timeout (or an error raised by another CTA) makes every role leave its
 // loop, in-flight copies are waited for, TMEM is released.
 #include <cudaTypedefs.h>
@@ -74,7 +75,7 @@ struct FLayout {
   static constexpr int EXTRA = (ATT_OFF + ATT_NEED > AFTER_STG) ? ((ATT_OFF + ATT_NEED - AFTER_STG + 1023) / 1024) * 1024 : 0;
   static constexpr int MISC_OFF = AFTER_STG + EXTRA;
   static constexpr int TOTAL = 1024 + MISC_OFF + C::MISC;
-  static_assert(C::SB * C::B_BYTES >= 8192 * 4, "a norm row (d <= 8192 floats) must fit in the activation ring");
+  static_assert(C::SB * C::B_BYTES >= 8192 * 4, "a final-norm row (d <= 8192 floats) must fit in the activation ring");
 };
 
 struct GP {
@@ -622,7 +623,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
   uint8_t* ringB = smem + LY::B_OFF;
   float* staging = reinterpret_cast<float*>(smem + LY::STG_OFF);
   uint8_t* att_smem = smem + LY::ATT_OFF;
-  float4* rowbuf = reinterpret_cast<float4*>(ringB);   // norm phases: one row, d <= 8192 floats
+  float4* rowbuf = reinterpret_cast<float4*>(ringB);   // final norm: one row, d <= 8192 floats
   uint64_t* fullA = reinterpret_cast<uint64_t*>(smem + LY::MISC_OFF);
   uint64_t* emptyA = fullA + C::SA;
   uint64_t* fullB = emptyA + C::SA;
@@ -828,7 +829,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1) fwd_kernel(const FwdParams p) 
     int nb = 0;   // grid barriers passed
     for (int ph = 0; ph < NP && ok; ++ph) {
       // which phase is this?
-      int kind, l = 0;   // 0 NORM0, 1 GEMM, 2 ATTN, 3 NORM (mlp), 4 NORM (next attn / final)
+      int kind, l = 0;   // 0 EMBED, 1 GEMM, 2 ATTN, 3 NORM (mlp, folded), 4 NORM (next attn: folded; final)
       int gi = -1;
       if (ph == 0) {
         kind = 0;
