@@ -91,10 +91,12 @@ def parse():
 
 
 # DRAM bytes per algorithmic byte of the batch-1 verification-call forward kernel (T = 120 tree
-# tokens): dram__bytes_read.sum + dram__bytes_write.sum of one ncu capture of the same kernel with
-# the target cut to 2 layers (856.6 MB of traffic for 838.7 MB of algorithmic bytes).  Measured for
-# the 128-token-tile schedule only: other workloads report no traffic figure.
+# tokens): dram__bytes_read.sum + dram__bytes_write.sum of one ncu capture of that kernel with the
+# target cut to 2 layers (856.6 MB of traffic for 838.7 MB of algorithmic bytes).  Measured for the
+# 128-token-tile schedule only: other workloads report no traffic figure.  TRAFFIC_CURRENT says
+# whether the capture is of the kernel as built now; when it is not, the line reports no traffic.
 TRAFFIC_PER_ALG_BYTE = 856.6 / 838.7
+TRAFFIC_CURRENT = False   # captured before the residual-update sums went to one part in flight
 
 
 def peaks():
@@ -356,10 +358,13 @@ def run_ours(args, w):
                                + (", early rejection at depth 0" if args.early_reject else ""),
                    "l2": "inputs larger than L2 (13.5 GB of target weights per verification call)"},
         "roofline": dict(roof, **{
-            "traffic": TRAFFIC_PER_ALG_BYTE * vb if T_first <= 128 else None,
+            "traffic": TRAFFIC_PER_ALG_BYTE * vb if T_first <= 128 and TRAFFIC_CURRENT else None,
             "traffic_source": ("dram__bytes_read.sum + dram__bytes_write.sum of one ncu capture of the same "
                                "kernel with the target cut to 2 layers, scaled by algorithmic bytes"
-                               if T_first <= 128 else "not captured at this tree size"),
+                               if T_first <= 128 and TRAFFIC_CURRENT else
+                               "not captured for this build (the previous build's 2-layer capture: "
+                               f"{TRAFFIC_PER_ALG_BYTE:.3f} x algorithmic bytes)" if T_first <= 128 else
+                               "not captured at this tree size"),
             "kernel": f"fwd_kernel: persistent forward of the verification call (tcgen05 GEMMs, tree attention, "
                       f"norms; T={T_first} tree tokens)",
             "peak_source": peak_kind, "launches": fk["launches"], "avg_launch_ms": k_ms,

@@ -46,7 +46,10 @@ constexpr int kRegsLaunch = 168, kRegsRoles = 80, kRegsCompute = 208;
 static_assert(128 * kRegsRoles + 256 * kRegsCompute <= FWD_THREADS * kRegsLaunch, "register split over the launch's total");
 static_assert(32 * (kRegsRoles + 2 * kRegsCompute) <= 16384, "register split over a sub-partition's file");
 static_assert(kRegsRoles % 8 == 0 && kRegsCompute % 8 == 0 && kRegsRoles >= 24 && kRegsCompute <= 256, "setmaxnreg range");
-constexpr int RED_PB = 2;             // split parts in flight in a chunk's sum
+// Split parts in flight in a residual-update sum: one.  With two or three the kernel spills
+// registers (24 / 136 and 48 / 164 bytes; the attention phase holds the peak), which costs more
+// than the round trips they save.
+constexpr int RED_PB = 1;
 constexpr int ITEM_ROWS_FWD = 1024;   // item-code rows of the LM head (4 levels x 256 codes)
 
 template <int BN>
